@@ -1,0 +1,196 @@
+/*
+ * aspis.h -- C ABI of libaspis, the GB300 (sm_103a) implementation of the
+ * parameter-server detection-and-aggregation step of Aspis
+ * (Konstantinidis & Ramamoorthy, "Aspis: Robust Detection for Distributed
+ * Learning", MLSys 2022).
+ *
+ * One training round at the PS (Algorithm 1): the K workers return, for each
+ * of the f = C(K,r) files, the r copies of that file's gradient (d floats).
+ * The PS
+ *   1. compares every pair of copies of every file          aspis_check
+ *   2. builds the agreement graph G (edge iff two workers
+ *      agree on all C(K-2,r-2) files they share)             aspis_check
+ *   3. finds the maximum cliques of G (Algorithm 3)           aspis_detect
+ *   4. picks one copy per file: an honest one when the
+ *      maximum clique is unique (Case 1), else the majority
+ *      copy (Case 2, Eq. 2)                                   aspis_select
+ *   5. aggregates the picked copies coordinate-wise
+ *      (lower median; mean optional)                          aspis_aggregate
+ *
+ * Conventions shared by every call:
+ *   - Pointers marked "device" are CUDA device pointers owned by the caller;
+ *     the library never allocates on the per-round path.  The only library
+ *     allocations are the tables of an aspis_assignment (host) and its device
+ *     mirror, released by aspis_assignment_free.
+ *   - Device calls are asynchronous on the given stream (a cudaStream_t
+ *     passed as void*; NULL = legacy default stream).  They return after the
+ *     launch; argument errors are returned synchronously before anything is
+ *     enqueued.  Outcomes decided on the device (clique-search budget, empty
+ *     selection) are written into the device-resident aspis_detection and are
+ *     visible after the stream is synchronized.
+ *   - Gradient copies are one fp32 buffer laid out [f][r][ld]: row (i, s) is
+ *     the vector returned by the worker in slot s of file i (slots are in
+ *     ascending worker order); only the first d of the ld floats of a row are
+ *     read.  ld >= d.  The 128-bit load path is used when the buffer is
+ *     16-byte aligned and ld % 4 == 0; otherwise a 4-byte path is used (not
+ *     an error).
+ *   - Equality of copies is bitwise equality of their fp32 words (+0 != -0;
+ *     NaNs equal iff their bit patterns are).
+ *   - Workers are 0-based.  Bit k of a worker mask is worker k.  K <= 31.
+ *   - Slot pairs (s,t), s<t, of one file are numbered (0,1),(0,2),...,
+ *     (0,r-1),(1,2),...,(r-2,r-1); bit p of a per-file mismatch word is set
+ *     iff the copies of the p-th pair differ.  r <= 8, so at most 28 bits.
+ */
+#ifndef ASPIS_H
+#define ASPIS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ASPIS_MAX_K 31
+#define ASPIS_MAX_R 8
+/* Largest number of files aspis_aggregate can reduce per coordinate (the
+ * per-coordinate working set is staged in shared memory). */
+#define ASPIS_MAX_AGG_FILES 6144
+
+typedef enum {
+    ASPIS_OK = 0,
+    ASPIS_E_INVAL = 1,           /* bad argument (NULL pointer, r<2, r>K, d<1, ld<d, mode) */
+    ASPIS_E_RANGE = 2,           /* K > 31, r > 8, or f > ASPIS_MAX_AGG_FILES for aggregation */
+    ASPIS_E_ALIGN = 3,           /* reserved: misalignment is handled, never reported */
+    ASPIS_E_CUDA = 4,            /* a CUDA runtime call or launch failed */
+    ASPIS_E_LIMIT = 5,           /* clique search ran out of its node budget (device status) */
+    ASPIS_E_EMPTY = 6,           /* no file kept a copy, nothing to aggregate (device status) */
+    ASPIS_E_NOT_IMPLEMENTED = 7
+} aspis_status;
+
+/* Subset-based file assignment (Algorithm 2; Example 1 fixes file 0 to the
+ * first r workers).  File i is given to the i-th r-subset of the workers in
+ * lexicographic order. */
+typedef struct {
+    int32_t K;                   /* workers */
+    int32_t r;                   /* redundancy: copies per file */
+    int64_t f;                   /* files, C(K,r) */
+    int64_t l;                   /* files per worker (computation load), C(K-1,r-1) */
+    int64_t pair_share;          /* files shared by any two workers, C(K-2,r-2) */
+    uint8_t *file_workers;       /* host [f*r]: worker of slot s of file i, ascending in s */
+    int32_t *worker_files;       /* host [K*l]: files of worker j, ascending */
+    uint8_t *slot_of;            /* host [K*l]: slot of worker j in worker_files[j*l+k] */
+    uint8_t *dev_file_workers;   /* device [f*r] mirror of file_workers, or NULL */
+} aspis_assignment;
+
+/* Outcome of detection and selection for one round; lives in device memory
+ * (the caller allocates sizeof(aspis_detection) bytes).  Written by
+ * aspis_detect (all but n_sel), aspis_select (n_sel) and aspis_aggregate
+ * (status = ASPIS_E_EMPTY when n_sel == 0). */
+typedef struct {
+    uint32_t clique_mask;        /* the maximum clique with the smallest mask value */
+    int32_t  omega;              /* size of a maximum clique */
+    uint32_t n_max_cliques;      /* number of maximum cliques */
+    int32_t  success;            /* 1 iff n_max_cliques == 1: H = clique (Case 1) */
+    int32_t  n_sel;              /* files whose copy enters aggregation */
+    int32_t  status;             /* ASPIS_OK, ASPIS_E_LIMIT or ASPIS_E_EMPTY */
+    uint32_t search_nodes;       /* Bron-Kerbosch nodes visited (diagnostic) */
+    uint32_t node_budget;        /* in: node limit per search branch, 0 = default
+                                    (2^20); read by aspis_detect, never written */
+} aspis_detection;
+
+/* Short text for a status code. */
+const char *aspis_status_str(int status);
+
+/* ABI version of this header (incremented on any signature change). */
+int aspis_abi_version(void);
+
+/* Algorithm 2.  Fills *out with host tables (allocated by the library).
+ * Requires 2 <= r <= K, K <= ASPIS_MAX_K, r <= ASPIS_MAX_R.  Host only: needs
+ * no GPU.  On error *out is zeroed. */
+aspis_status aspis_assign(int K, int r, aspis_assignment *out);
+
+/* Uploads file_workers to a device mirror (cudaMalloc + copy, synchronous),
+ * once; later calls are no-ops.  Needed by every device call below. */
+aspis_status aspis_assignment_to_device(aspis_assignment *a);
+
+/* Frees the host tables and the device mirror and zeroes *a. */
+void aspis_assignment_free(aspis_assignment *a);
+
+/* Steps 1-2: per-file agreement alpha_i and graph G (Section 4, the
+ * definitions of alpha_i^{(j1,j2)} and alpha^{(j1,j2)} and the edge rule of
+ * Algorithm 3).
+ *   copies    device [f][r][ld] fp32
+ *   file_neq  device [f] uint32, out: per-file slot-pair mismatch word
+ *   adj       device [K] uint32, out: adj[j] bit k = edge (j,k), i.e. workers
+ *             j and k returned bitwise-equal copies for every file they share;
+ *             no self loops, bits >= K zero
+ * Reads f*r*d*4 bytes.  Overwrites file_neq and adj entirely. */
+aspis_status aspis_check(const float *copies, int64_t d, int64_t ld,
+                         const aspis_assignment *a, uint32_t *file_neq,
+                         uint32_t *adj, void *stream);
+
+/* Step 3: all maximum cliques of G (Algorithm 3: every maximum clique is
+ * listed; exactly one of them means successful detection).  Bron-Kerbosch with pivoting over
+ * 32-bit vertex masks in one thread block; each search branch has a node
+ * budget (det->node_budget, 0 = 2^20 nodes) after which det->status =
+ * ASPIS_E_LIMIT and det->success = 0 (the round then falls back to majority
+ * voting, Case 2).
+ *   adj  device [K] uint32 (as written by aspis_check)
+ *   det  device aspis_detection, out (n_sel reset to 0) */
+aspis_status aspis_detect(const uint32_t *adj, int K, aspis_detection *det,
+                          void *stream);
+
+/* Step 4: one copy per file (Algorithm 1).
+ *   Case 1 (det->success): the copy of the lowest slot whose worker is in the
+ *     clique; -1 (file dropped) if the file has no such worker.
+ *   Case 2: the majority copy m_i of Eq. 2, read as the largest class of
+ *     bitwise-equal copies (ties to the class holding the lower slot); sel is
+ *     that class's lowest slot.  No file is dropped.
+ *   file_neq  device [f] (from aspis_check)
+ *   det       device, in: success/clique_mask; out: n_sel (added to)
+ *   sel       device [f] int8, out: chosen slot or -1 */
+aspis_status aspis_select(const uint32_t *file_neq, aspis_detection *det,
+                          const aspis_assignment *a, int8_t *sel, void *stream);
+
+/* Step 5: coordinate-wise aggregation of the chosen copies (Algorithm 1:
+ * median of the majority gradients in Case 2, mean in Case 1).
+ *   mode 0: lower median: for each coordinate c < d the element of rank
+ *           floor((n_sel-1)/2) of {copies[i][sel[i]][c] : sel[i] >= 0} in
+ *           IEEE-754 totalOrder; out[c] has that element's exact bits.
+ *   mode 1: mean of the same values (compensated fp32 summation, one final
+ *           rounding; within 1e-6 relative of the exactly-rounded mean).
+ *   sel   device [f] (from aspis_select)
+ *   det   device; n_sel is read, status set to ASPIS_E_EMPTY when 0 (then
+ *         out is left untouched)
+ *   out   device [d] fp32
+ * Reads n_sel*d*4 bytes and writes d*4.  f must be <= ASPIS_MAX_AGG_FILES. */
+aspis_status aspis_aggregate(const float *copies, int64_t d, int64_t ld,
+                             const aspis_assignment *a, const int8_t *sel,
+                             aspis_detection *det, int mode, float *out,
+                             void *stream);
+
+/* Steps 1-5 back to back on one stream (the whole PS step of one round). */
+aspis_status aspis_round(const float *copies, int64_t d, int64_t ld,
+                         const aspis_assignment *a, uint32_t *file_neq,
+                         uint32_t *adj, aspis_detection *det, int8_t *sel,
+                         int mode, float *out, void *stream);
+
+/* The whole round from host memory: copies the f*r*ld floats at
+ * host_copies (pinned memory gives full bandwidth) into the device buffer
+ * dev_copies, runs aspis_round, and copies the d aggregated floats into
+ * host_out and the detection record into host_det.  All work and copies are
+ * enqueued on the stream; the host buffers must stay valid until it is
+ * synchronized.  Device buffers are the caller's, as for aspis_round. */
+aspis_status aspis_round_host(const float *host_copies, float *dev_copies,
+                              int64_t d, int64_t ld, const aspis_assignment *a,
+                              uint32_t *file_neq, uint32_t *adj,
+                              aspis_detection *det, int8_t *sel, int mode,
+                              float *dev_out, float *host_out,
+                              aspis_detection *host_det, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ASPIS_H */

@@ -1,0 +1,252 @@
+"""Python binding of libaspis (C ABI in ``include/aspis.h``).
+
+Argument marshalling only: every step of the PS round runs in the library's
+CUDA kernels.  PyTorch supplies device memory and streams.  There is no CPU
+fallback; if ``libaspis.so`` is missing, importing the binding raises.
+Build it with ``python paper_2108_02416_gb300/build.py`` (or
+``__graft_entry__.build()``).
+
+The call names mirror the C entry points:
+
+  aspis_assign(K, r) -> Assignment          Algorithm 2
+  aspis_check(copies, d, a, file_neq, adj)  per-file agreement + graph G
+  aspis_detect(adj, K, det)                 Algorithm 3 (maximum cliques)
+  aspis_select(file_neq, det, a, sel)       Algorithm 1 (Case 1 / Case 2)
+  aspis_aggregate(copies, d, a, sel, det, out, mode)   coordinate-wise median / mean
+  aspis_round(...)                          the four device steps on one stream
+  aspis_round_host(...)                     the same from pinned host memory
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "libaspis.so")
+
+OK, E_INVAL, E_RANGE, E_ALIGN, E_CUDA, E_LIMIT, E_EMPTY, E_NOT_IMPLEMENTED = range(8)
+MAX_K, MAX_R, MAX_AGG_FILES = 31, 8, 6144
+MEDIAN, MEAN = 0, 1
+
+
+class AspisError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_str(status)} ({status})")
+
+
+class _Assignment(ctypes.Structure):
+    _fields_ = [("K", ctypes.c_int32), ("r", ctypes.c_int32), ("f", ctypes.c_int64),
+                ("l", ctypes.c_int64), ("pair_share", ctypes.c_int64),
+                ("file_workers", ctypes.POINTER(ctypes.c_uint8)),
+                ("worker_files", ctypes.POINTER(ctypes.c_int32)),
+                ("slot_of", ctypes.POINTER(ctypes.c_uint8)),
+                ("dev_file_workers", ctypes.c_void_p)]
+
+
+class Detection(ctypes.Structure):
+    """Host image of ``aspis_detection`` (32 bytes)."""
+    _fields_ = [("clique_mask", ctypes.c_uint32), ("omega", ctypes.c_int32),
+                ("n_max_cliques", ctypes.c_uint32), ("success", ctypes.c_int32),
+                ("n_sel", ctypes.c_int32), ("status", ctypes.c_int32),
+                ("search_nodes", ctypes.c_uint32), ("node_budget", ctypes.c_uint32)]
+
+    @classmethod
+    def from_tensor(cls, t):
+        """Read a device/host uint8[32] tensor holding an aspis_detection."""
+        raw = bytes(t.detach().to("cpu").contiguous().numpy().tobytes())
+        return cls.from_buffer_copy(raw)
+
+    def as_dict(self):
+        return {k: getattr(self, k) for k, _ in self._fields_}
+
+
+DETECTION_BYTES = ctypes.sizeof(Detection)
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build it first (python "
+                          "paper_2108_02416_gb300/build.py or __graft_entry__.build()); "
+                          "there is no CPU fallback")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
+    A = ctypes.POINTER(_Assignment)
+    sig = {
+        "aspis_status_str": ([i32], ctypes.c_char_p),
+        "aspis_abi_version": ([], i32),
+        "aspis_assign": ([i32, i32, A], i32),
+        "aspis_assignment_to_device": ([A], i32),
+        "aspis_assignment_free": ([A], None),
+        "aspis_check": ([P, i64, i64, A, P, P, P], i32),
+        "aspis_detect": ([P, i32, P, P], i32),
+        "aspis_select": ([P, P, A, P, P], i32),
+        "aspis_aggregate": ([P, i64, i64, A, P, P, i32, P, P], i32),
+        "aspis_round": ([P, i64, i64, A, P, P, P, P, i32, P, P], i32),
+        "aspis_round_host": ([P, P, i64, i64, A, P, P, P, P, i32, P, P, P, P], i32),
+    }
+    for name, (args, res) in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = res
+    return lib
+
+
+lib = _load()
+
+
+def status_str(status: int) -> str:
+    return lib.aspis_status_str(int(status)).decode()
+
+
+def _ok(status: int, where: str):
+    if status != OK:
+        raise AspisError(status, where)
+
+
+class Assignment:
+    """Owns an ``aspis_assignment`` (host tables + device mirror)."""
+
+    def __init__(self, K: int, r: int, device: bool = True):
+        self._a = _Assignment()
+        _ok(lib.aspis_assign(K, r, ctypes.byref(self._a)), "aspis_assign")
+        if device:
+            self.to_device()
+
+    def to_device(self):
+        _ok(lib.aspis_assignment_to_device(ctypes.byref(self._a)), "aspis_assignment_to_device")
+        return self
+
+    @property
+    def ref(self):
+        return ctypes.byref(self._a)
+
+    K = property(lambda s: s._a.K)
+    r = property(lambda s: s._a.r)
+    f = property(lambda s: s._a.f)
+    l = property(lambda s: s._a.l)
+    pair_share = property(lambda s: s._a.pair_share)
+
+    def file_workers(self):
+        import numpy as np
+        return np.ctypeslib.as_array(self._a.file_workers, (self.f * self.r,)).reshape(self.f, self.r).copy()
+
+    def worker_files(self):
+        import numpy as np
+        return np.ctypeslib.as_array(self._a.worker_files, (self.K * self.l,)).reshape(self.K, self.l).copy()
+
+    def slot_of(self):
+        import numpy as np
+        return np.ctypeslib.as_array(self._a.slot_of, (self.K * self.l,)).reshape(self.K, self.l).copy()
+
+    def close(self):
+        if getattr(self, "_a", None) is not None and self._a.K:
+            lib.aspis_assignment_free(ctypes.byref(self._a))
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def aspis_assign(K: int, r: int, device: bool = True) -> Assignment:
+    return Assignment(K, r, device)
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return ctypes.c_void_p(stream)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dev(t, dtype=None, name="tensor"):
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _ld(copies, a: Assignment):
+    if copies.dim() != 3 or copies.shape[0] != a.f or copies.shape[1] != a.r:
+        raise ValueError(f"copies must be [f={a.f}, r={a.r}, ld], got {tuple(copies.shape)}")
+    return int(copies.shape[2])
+
+
+def aspis_check(copies, d: int, a: Assignment, file_neq, adj, stream=None):
+    import torch
+    ld = _ld(copies, a)
+    _ok(lib.aspis_check(_dev(copies, torch.float32, "copies"), d, ld, a.ref,
+                        _dev(file_neq, torch.int32, "file_neq"), _dev(adj, torch.int32, "adj"),
+                        _stream(stream)), "aspis_check")
+
+
+def aspis_detect(adj, K: int, det, stream=None):
+    import torch
+    _ok(lib.aspis_detect(_dev(adj, torch.int32, "adj"), K, _dev(det, torch.uint8, "det"),
+                         _stream(stream)), "aspis_detect")
+
+
+def aspis_select(file_neq, det, a: Assignment, sel, stream=None):
+    import torch
+    _ok(lib.aspis_select(_dev(file_neq, torch.int32, "file_neq"), _dev(det, torch.uint8, "det"),
+                         a.ref, _dev(sel, torch.int8, "sel"), _stream(stream)), "aspis_select")
+
+
+def aspis_aggregate(copies, d: int, a: Assignment, sel, det, out, mode: int = MEDIAN, stream=None):
+    import torch
+    ld = _ld(copies, a)
+    _ok(lib.aspis_aggregate(_dev(copies, torch.float32, "copies"), d, ld, a.ref,
+                            _dev(sel, torch.int8, "sel"), _dev(det, torch.uint8, "det"), mode,
+                            _dev(out, torch.float32, "out"), _stream(stream)), "aspis_aggregate")
+
+
+def aspis_round(copies, d: int, a: Assignment, file_neq, adj, det, sel, out, mode: int = MEDIAN,
+                stream=None):
+    import torch
+    ld = _ld(copies, a)
+    _ok(lib.aspis_round(_dev(copies, torch.float32, "copies"), d, ld, a.ref,
+                        _dev(file_neq, torch.int32, "file_neq"), _dev(adj, torch.int32, "adj"),
+                        _dev(det, torch.uint8, "det"), _dev(sel, torch.int8, "sel"), mode,
+                        _dev(out, torch.float32, "out"), _stream(stream)), "aspis_round")
+
+
+def aspis_round_host(host_copies, dev_copies, d: int, a: Assignment, file_neq, adj, det, sel,
+                     dev_out, host_out, host_det, mode: int = MEDIAN, stream=None):
+    """host_copies / host_out / host_det: CPU tensors (pinned for full speed)."""
+    import torch
+    ld = _ld(dev_copies, a)
+    for t, nm in ((host_copies, "host_copies"), (host_out, "host_out"), (host_det, "host_det")):
+        if t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{nm} must be a contiguous CPU tensor")
+    if host_copies.numel() != dev_copies.numel() or host_copies.dtype != torch.float32:
+        raise ValueError("host_copies must match dev_copies (float32)")
+    _ok(lib.aspis_round_host(ctypes.c_void_p(host_copies.data_ptr()),
+                             _dev(dev_copies, torch.float32, "dev_copies"), d, ld, a.ref,
+                             _dev(file_neq, torch.int32, "file_neq"), _dev(adj, torch.int32, "adj"),
+                             _dev(det, torch.uint8, "det"), _dev(sel, torch.int8, "sel"), mode,
+                             _dev(dev_out, torch.float32, "dev_out"),
+                             ctypes.c_void_p(host_out.data_ptr()),
+                             ctypes.c_void_p(host_det.data_ptr()), _stream(stream)),
+        "aspis_round_host")
+
+
+class RoundBuffers:
+    """Device buffers of one round for an assignment (allocated by torch)."""
+
+    def __init__(self, a: Assignment, d: int, device="cuda"):
+        import torch
+        self.file_neq = torch.zeros(a.f, dtype=torch.int32, device=device)
+        self.adj = torch.zeros(a.K, dtype=torch.int32, device=device)
+        self.det = torch.zeros(DETECTION_BYTES, dtype=torch.uint8, device=device)
+        self.sel = torch.zeros(a.f, dtype=torch.int8, device=device)
+        self.out = torch.zeros(d, dtype=torch.float32, device=device)
+
+    def detection(self) -> Detection:
+        return Detection.from_tensor(self.det)

@@ -1,0 +1,173 @@
+// C-ABI entry points of libaspis: argument checks, then the kernel launches
+// of check.cu, detect.cu and aggregate.cu on the caller's stream.
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "aspis_internal.cuh"
+
+namespace aspis {
+
+size_t aggregate_smem_bytes(int64_t f, int *tc_out);
+
+int sm_count()
+{
+    static std::mutex mu;
+    static int cached[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev < 0 || dev >= 64) dev = 0;
+    std::lock_guard<std::mutex> g(mu);
+    if (!cached[dev]) {
+        int n = 0;
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        cached[dev] = n > 0 ? n : 1;
+    }
+    return cached[dev];
+}
+
+}  // namespace aspis
+
+using namespace aspis;
+
+namespace {
+
+inline aspis_status cuda_status(cudaError_t e) { return e == cudaSuccess ? ASPIS_OK : ASPIS_E_CUDA; }
+
+aspis_status check_assignment(const aspis_assignment *a)
+{
+    if (!a || !a->dev_file_workers) return ASPIS_E_INVAL;
+    if (a->r < 2 || a->K < a->r || a->f < 1) return ASPIS_E_INVAL;
+    if (a->K > ASPIS_MAX_K || a->r > ASPIS_MAX_R) return ASPIS_E_RANGE;
+    return ASPIS_OK;
+}
+
+aspis_status check_copies(const float *copies, int64_t d, int64_t ld, const aspis_assignment *a)
+{
+    if (!copies || d < 1 || ld < d) return ASPIS_E_INVAL;
+    // every element index i*r*ld + s*ld + c must fit in int64
+    const int64_t rows = a->f * a->r;
+    if (ld > (int64_t)(INT64_MAX / 8) / rows) return ASPIS_E_RANGE;
+    return ASPIS_OK;
+}
+
+}  // namespace
+
+extern "C" aspis_status aspis_assignment_to_device(aspis_assignment *a)
+{
+    if (!a || !a->file_workers || a->f < 1 || a->r < 2) return ASPIS_E_INVAL;
+    if (a->dev_file_workers) return ASPIS_OK;
+    uint8_t *p = nullptr;
+    const size_t bytes = (size_t)(a->f * a->r);
+    if (cudaMalloc(&p, bytes) != cudaSuccess) return ASPIS_E_CUDA;
+    if (cudaMemcpy(p, a->file_workers, bytes, cudaMemcpyHostToDevice) != cudaSuccess) {
+        cudaFree(p);
+        return ASPIS_E_CUDA;
+    }
+    a->dev_file_workers = p;
+    return ASPIS_OK;
+}
+
+extern "C" void aspis_assignment_free(aspis_assignment *a)
+{
+    if (!a) return;
+    std::free(a->file_workers);
+    std::free(a->worker_files);
+    std::free(a->slot_of);
+    if (a->dev_file_workers) cudaFree(a->dev_file_workers);
+    std::memset(a, 0, sizeof(*a));
+}
+
+extern "C" aspis_status aspis_check(const float *copies, int64_t d, int64_t ld,
+                                    const aspis_assignment *a, uint32_t *file_neq,
+                                    uint32_t *adj, void *stream)
+{
+    aspis_status s = check_assignment(a);
+    if (s != ASPIS_OK) return s;
+    if ((s = check_copies(copies, d, ld, a)) != ASPIS_OK) return s;
+    if (!file_neq || !adj) return ASPIS_E_INVAL;
+    cudaStream_t st = (cudaStream_t)stream;
+    if (cudaMemsetAsync(file_neq, 0, sizeof(uint32_t) * (size_t)a->f, st) != cudaSuccess)
+        return ASPIS_E_CUDA;
+    if ((s = cuda_status(launch_compare(copies, a->f, a->r, d, ld, file_neq, st))) != ASPIS_OK)
+        return s;
+    return cuda_status(launch_graph(file_neq, a->dev_file_workers, a->f, a->r, a->K, adj, st));
+}
+
+extern "C" aspis_status aspis_detect(const uint32_t *adj, int K, aspis_detection *det,
+                                     void *stream)
+{
+    if (!adj || !det) return ASPIS_E_INVAL;
+    if (K < 2) return ASPIS_E_INVAL;
+    if (K > ASPIS_MAX_K) return ASPIS_E_RANGE;
+    return cuda_status(launch_detect(adj, K, det, (cudaStream_t)stream));
+}
+
+extern "C" aspis_status aspis_select(const uint32_t *file_neq, aspis_detection *det,
+                                     const aspis_assignment *a, int8_t *sel, void *stream)
+{
+    aspis_status s = check_assignment(a);
+    if (s != ASPIS_OK) return s;
+    if (!file_neq || !det || !sel) return ASPIS_E_INVAL;
+    return cuda_status(launch_select(file_neq, det, a->dev_file_workers, a->f, a->r, sel,
+                                     (cudaStream_t)stream));
+}
+
+extern "C" aspis_status aspis_aggregate(const float *copies, int64_t d, int64_t ld,
+                                        const aspis_assignment *a, const int8_t *sel,
+                                        aspis_detection *det, int mode, float *out,
+                                        void *stream)
+{
+    aspis_status s = check_assignment(a);
+    if (s != ASPIS_OK) return s;
+    if ((s = check_copies(copies, d, ld, a)) != ASPIS_OK) return s;
+    if (!sel || !det || !out || (mode != 0 && mode != 1)) return ASPIS_E_INVAL;
+    if (a->f > ASPIS_MAX_AGG_FILES) return ASPIS_E_RANGE;
+    int tc = 0;
+    if (!aggregate_smem_bytes(a->f, &tc) || !tc) return ASPIS_E_RANGE;
+    return cuda_status(launch_aggregate(copies, a->f, a->r, d, ld, sel, det, mode, out,
+                                        (cudaStream_t)stream));
+}
+
+extern "C" aspis_status aspis_round(const float *copies, int64_t d, int64_t ld,
+                                    const aspis_assignment *a, uint32_t *file_neq,
+                                    uint32_t *adj, aspis_detection *det, int8_t *sel,
+                                    int mode, float *out, void *stream)
+{
+    aspis_status s = check_assignment(a);
+    if (s != ASPIS_OK) return s;
+    if ((s = check_copies(copies, d, ld, a)) != ASPIS_OK) return s;
+    if (!file_neq || !adj || !det || !sel || !out || (mode != 0 && mode != 1))
+        return ASPIS_E_INVAL;
+    if (a->f > ASPIS_MAX_AGG_FILES) return ASPIS_E_RANGE;
+    if ((s = aspis_check(copies, d, ld, a, file_neq, adj, stream)) != ASPIS_OK) return s;
+    if ((s = aspis_detect(adj, a->K, det, stream)) != ASPIS_OK) return s;
+    if ((s = aspis_select(file_neq, det, a, sel, stream)) != ASPIS_OK) return s;
+    return aspis_aggregate(copies, d, ld, a, sel, det, mode, out, stream);
+}
+
+extern "C" aspis_status aspis_round_host(const float *host_copies, float *dev_copies,
+                                         int64_t d, int64_t ld, const aspis_assignment *a,
+                                         uint32_t *file_neq, uint32_t *adj,
+                                         aspis_detection *det, int8_t *sel, int mode,
+                                         float *dev_out, float *host_out,
+                                         aspis_detection *host_det, void *stream)
+{
+    aspis_status s = check_assignment(a);
+    if (s != ASPIS_OK) return s;
+    if (!host_copies || !host_out || !host_det) return ASPIS_E_INVAL;
+    if ((s = check_copies(dev_copies, d, ld, a)) != ASPIS_OK) return s;
+    cudaStream_t st = (cudaStream_t)stream;
+    const size_t bytes = sizeof(float) * (size_t)(a->f * a->r) * (size_t)ld;
+    if (cudaMemcpyAsync(dev_copies, host_copies, bytes, cudaMemcpyHostToDevice, st) != cudaSuccess)
+        return ASPIS_E_CUDA;
+    s = aspis_round(dev_copies, d, ld, a, file_neq, adj, det, sel, mode, dev_out, stream);
+    if (s != ASPIS_OK) return s;
+    if (cudaMemcpyAsync(host_out, dev_out, sizeof(float) * (size_t)d, cudaMemcpyDeviceToHost,
+                        st) != cudaSuccess)
+        return ASPIS_E_CUDA;
+    if (cudaMemcpyAsync(host_det, det, sizeof(aspis_detection), cudaMemcpyDeviceToHost, st) !=
+        cudaSuccess)
+        return ASPIS_E_CUDA;
+    return ASPIS_OK;
+}
