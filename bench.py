@@ -1,0 +1,391 @@
+"""Benchmark of the Aspis PS detection-and-aggregation step on GB300.
+
+One step = one PS round on one GPU: aspis_check (compare every copy pair of
+every file, build G), aspis_detect (maximum cliques), aspis_select (one copy
+per file) and aspis_aggregate (coordinate-wise lower median), all on one
+stream, over synthetic copies already resident in HBM.
+
+Default workload: K=15 workers, r=3, f=455 files, d=11,173,962 fp32 (a
+flattened ResNet-18 gradient), optimal (strong) attack with q=3 colluding
+ALIE adversaries: 61.0 GB of copies, larger than L2, so no flush is needed
+between rounds.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME]
+    python bench.py --impl reference ...    # the CPU oracle on a bounded slice
+
+Prints one JSON line (rank 0).  With N > 1 (torchrun) every rank runs an
+independent replica on its own GPU; there is no data-path collective.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+DEFAULT_CONFIG = "k15_r3_d11m_strong_alie"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    p.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(synth.CONFIGS))
+    p.add_argument("--mode", type=int, default=0, help="0 = lower median, 1 = mean")
+    p.add_argument("--e2e-steps", type=int, default=5)
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=12.0,
+                   help="target CPU time of the oracle baseline sample")
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            pk = json.load(fh)
+        return float(pk["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def algorithmic_bytes(w, n_sel):
+    f = w.f
+    cmp_bytes = f * w.r * w.d * 4                  # every copy read once
+    agg_bytes = n_sel * w.d * 4 + w.d * 4          # chosen copies read, d written
+    return cmp_bytes, agg_bytes
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while timing."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        try:
+            for line in open(self.path):
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9 and parts[1].replace(".", "").isdigit():
+                    rows.append(parts)
+        except Exception:
+            pass
+        finally:
+            if self.path and os.path.exists(self.path):
+                os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        sm = [float(r[1]) for r in rows]
+        mx = max(float(r[2]) for r in rows)
+        load = [s for s, r in zip(sm, rows) if float(r[3] or 0) > 300.0] or sm
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for r in rows for k in range(4) if r[5 + k].lower() == "active"})
+        return {"sm_mhz": statistics.median(load), "sm_max_mhz": mx, "reasons": reasons,
+                "samples": len(rows), "power_w_max": max(float(r[3] or 0) for r in rows)}
+
+
+def profile_traffic(kernel_tag: str, workload: str, units: int, source: str):
+    """dram bytes per launch from a committed ncu summary, scaled to `units`,
+    or None when the summary is absent or older than the kernel source."""
+    pdir = os.path.join(ROOT, "profiles")
+    sha = hashlib.sha256(open(source, "rb").read()).hexdigest()[:16]
+    pat = re.compile(rf"^bench-traffic: {re.escape(kernel_tag)} workload=(\S+) "
+                     r"units=(\d+) dram_bytes=(\d+) source_sha=(\w+)")
+    if not os.path.isdir(pdir):
+        return None
+    for fn in sorted(os.listdir(pdir)):
+        if not fn.endswith((".md", ".txt")):
+            continue
+        for line in open(os.path.join(pdir, fn)):
+            m = pat.match(line.strip())
+            if m and m.group(4) == sha:
+                u, b = int(m.group(2)), int(m.group(3))
+                return int(round(b * units / u))
+    return None
+
+
+def json_line(obj):
+    print(json.dumps(obj), flush=True)
+
+
+# --------------------------------------------------------------- CPU oracle
+
+
+def oracle_sample(w, file_workers, ds, host_slice=None, nthreads=None):
+    """Times the oracle on coordinates [0, ds) of all copies; returns
+    (seconds, RoundResult)."""
+    import oracle
+    import numpy as np
+    if host_slice is None:
+        host_slice = synth.build_copies_np(w, file_workers, 0, ds)
+    a = oracle.assign(w.K, w.r)
+    assert np.array_equal(a.file_workers, file_workers)
+    t0 = time.perf_counter()
+    res = oracle.run_round(host_slice, a, ds, 0, nthreads)
+    return time.perf_counter() - t0, res
+
+
+def run_reference(args, w):
+    """--impl reference: the oracle as it stands on the host cores."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import oracle
+    cores = os.cpu_count() or 1
+    a = oracle.assign(w.K, w.r)
+    # size the slice so that warmup + steps fit in about two minutes
+    probe = 8192
+    t_probe, _ = oracle_sample(w, a.file_workers, probe)
+    per_step = max(0.5, 90.0 / max(1, args.steps + args.warmup))
+    # the slice is also generated on the host, so it stays at most 128 Ki coordinates
+    ds = int(min(w.d, 131072, max(probe, probe * per_step / max(t_probe, 1e-3))))
+    host = synth.build_copies_np(w, a.file_workers, 0, ds)
+    for _ in range(args.warmup):
+        oracle_sample(w, a.file_workers, ds, host)
+    times = [oracle_sample(w, a.file_workers, ds, host)[0] for _ in range(args.steps)]
+    ms = statistics.mean(times) * 1e3 * (w.d / ds)
+    sample = (f"coordinates [0, {ds}) of all {w.f}x{w.r} copies per step (check, detect, "
+              f"select, lower median); ms/round scaled by d/{ds}")
+    json_line({
+        "impl": "reference", "metric": metric_name(w), "value": ms, "unit": "ms/round",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms, "higher_is_better": False, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": config_obj(w, args),
+        "cpu_baseline": {"value": ms, "unit": "ms/round", "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": ms, "unit": "ms/round", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    })
+
+
+def metric_name(w):
+    return f"PS detect+aggregate ms/round (K={w.K}, r={w.r}, d={w.d})"
+
+
+def config_obj(w, args):
+    return {"workload": w.name, "K": w.K, "r": w.r, "f": w.f, "d": w.d, "ld": w.ld, "q": w.q,
+            "attack": w.attack, "distortion": w.distortion,
+            "aggregator": "lower_median" if args.mode == 0 else "mean",
+            "l2": "inputs larger than L2 (no flush)" if w.f * w.r * w.d * 4 > 200e6
+            else "L2 flushed between steps",
+            "parallelism": f"replicas x{args.gpus}"}
+
+
+# --------------------------------------------------------------- GPU arm
+
+
+def main():
+    args = parse()
+    w = synth.CONFIGS[args.config]
+    if args.impl == "reference":
+        return run_reference(args, w)
+
+    import numpy as np
+    import torch
+    import paper_2108_02416_gb300 as ap
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    a = ap.aspis_assign(w.K, w.r)
+    fw = a.file_workers()
+    copies = synth.build_copies_torch(w, fw, dev)
+    buf = ap.RoundBuffers(a, w.d, dev)
+    stream = torch.cuda.Stream(device=dev)
+    small = w.f * w.r * w.d * 4 <= 200e6
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev) if small else None
+
+    def one_round(ev=None):
+        if flush is not None:
+            flush.zero_()
+        if ev:
+            ev[0].record(stream)
+        ap.aspis_check(copies, w.d, a, buf.file_neq, buf.adj, stream)
+        if ev:
+            ev[1].record(stream)
+        ap.aspis_detect(buf.adj, w.K, buf.det, stream)
+        ap.aspis_select(buf.file_neq, buf.det, a, buf.sel, stream)
+        if ev:
+            ev[2].record(stream)
+        ap.aspis_aggregate(copies, w.d, a, buf.sel, buf.det, buf.out, args.mode, stream)
+        if ev:
+            ev[3].record(stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            one_round()
+    torch.cuda.synchronize()
+    det = buf.detection()
+    if det.status != ap.OK:
+        raise RuntimeError(f"round status {ap.status_str(det.status)}")
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t_start.record(stream)
+        for k in range(args.steps):
+            one_round(evs[k])
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    if flush is not None:         # small inputs: exclude the L2 flush kernels
+        total_ms = sum(e[0].elapsed_time(e[3]) for e in evs)
+    if dist:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    clocks = clk.summary()
+    check_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    detsel_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    agg_ms = [e[2].elapsed_time(e[3]) for e in evs]
+
+    n_sel = buf.detection().n_sel
+    cmp_bytes, agg_bytes = algorithmic_bytes(w, n_sel)
+    peak, peak_kind = peaks()
+    ms_round = total_ms / (args.steps * world)
+    cmp_gbs = cmp_bytes / (statistics.mean(check_ms) * 1e-3) / 1e9
+    agg_gbs = agg_bytes / (statistics.mean(agg_ms) * 1e-3) / 1e9
+    all_gbs = (cmp_bytes + agg_bytes) / (total_ms / args.steps * 1e-3) / 1e9
+    csrc = os.path.join(ROOT, "paper_2108_02416_gb300", "csrc")
+    cmp_traffic = profile_traffic("compare_vec_kernel", w.name, w.f * w.r * w.d,
+                                  os.path.join(csrc, "check.cu"))
+    agg_traffic = profile_traffic("aggregate_kernel", w.name, n_sel * w.d,
+                                  os.path.join(csrc, "aggregate.cu"))
+
+    # ---- end to end through aspis_round_host from pinned host memory
+    e2e = None
+    if not args.no_e2e:
+        host = torch.empty(copies.shape, dtype=torch.float32, pin_memory=True)
+        host.copy_(copies)
+        hout = torch.empty(w.d, dtype=torch.float32, pin_memory=True)
+        hdet = torch.zeros(ap.DETECTION_BYTES, dtype=torch.uint8, pin_memory=True)
+        ap.aspis_round_host(host, copies, w.d, a, buf.file_neq, buf.adj, buf.det, buf.sel,
+                            buf.out, hout, hdet, args.mode, stream)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.e2e_steps):
+            ap.aspis_round_host(host, copies, w.d, a, buf.file_neq, buf.adj, buf.det, buf.sel,
+                                buf.out, hout, hdet, args.mode, stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = e0.elapsed_time(e1) / args.e2e_steps
+        ok = np.array_equal(hout.numpy().view(np.uint32), buf.out.cpu().numpy().view(np.uint32))
+        e2e = {"value": e2e_ms / world, "unit": "ms/round", "steps": args.e2e_steps,
+               "h2d_bytes_per_step": int(host.numel() * 4),
+               "d2h_bytes_per_step": int(w.d * 4 + ap.DETECTION_BYTES),
+               "output_matches_device_run": bool(ok)}
+        del host
+
+    # ---- CPU baseline: the oracle on a bounded slice of the same copies
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        probe = 4096
+        hs = copies[:, :, :probe].contiguous().cpu().numpy()
+        tp, _ = oracle_sample(w, fw, probe, hs)
+        ds = int(min(w.d, 2_000_000, max(probe, probe * args.cpu_seconds / max(tp, 1e-3))))
+        hs = copies[:, :, :ds].contiguous().cpu().numpy()
+        ts, res = oracle_sample(w, fw, ds, hs)
+        cores = os.cpu_count() or 1
+        cpu = {"value": ts * 1e3 * (w.d / ds), "unit": "ms/round", "cores": cores,
+               "kind": "oracle",
+               "sample": f"coordinates [0, {ds}) of all {w.f}x{w.r} copies (check, detect, "
+                         f"select, lower median on the slice, {ts:.1f} s); ms/round scaled "
+                         f"by d/{ds}",
+               "agrees_with_gpu_on_slice": bool(np.array_equal(
+                   res.out.view(np.uint32), buf.out[:ds].cpu().numpy().view(np.uint32))
+                   if res.out is not None and args.mode == 0 else None)}
+
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return
+    launches_per_round = 5    # compare, graph, detect, select, aggregate
+    line = {
+        "metric": metric_name(w), "value": ms_round, "unit": "ms/round", "n_gpus": world,
+        "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": total_ms / args.steps,
+        "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded counter-based generator; paper workload shapes)",
+        "config": config_obj(w, args),
+        "gbps": all_gbs,
+        "roofline": {"bound": "hbm", "kernel": "compare (aspis_check)",
+                     "achieved": cmp_gbs, "peak": peak, "unit": "GB/s",
+                     "frac": cmp_gbs / peak, "peak_kind": peak_kind,
+                     "traffic": cmp_traffic, "algorithmic_bytes": cmp_bytes},
+        "roofline_aggregate": {"bound": "hbm", "kernel": "aggregate (lower median)",
+                               "achieved": agg_gbs, "peak": peak, "unit": "GB/s",
+                               "frac": agg_gbs / peak, "peak_kind": peak_kind,
+                               "traffic": agg_traffic, "algorithmic_bytes": agg_bytes,
+                               "ms": statistics.mean(agg_ms)},
+        "passes_ms": {"check": statistics.mean(check_ms),
+                      "detect_select": statistics.mean(detsel_ms),
+                      "aggregate": statistics.mean(agg_ms)},
+        "detection": {"omega": det.omega, "n_max_cliques": det.n_max_cliques,
+                      "success": det.success, "n_sel": n_sel},
+        "clocks": clocks,
+        "gpu_launches": launches_per_round * args.steps,
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    json_line(line)
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
