@@ -46,6 +46,8 @@ def parse():
     p.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     p.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(synth.CONFIGS))
     p.add_argument("--mode", type=int, default=0, help="0 = lower median, 1 = mean")
+    p.add_argument("--d", type=int, default=0,
+                   help="override the gradient length (smaller cases for profiling)")
     p.add_argument("--e2e-steps", type=int, default=5)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
@@ -219,6 +221,9 @@ def config_obj(w, args):
 def main():
     args = parse()
     w = synth.CONFIGS[args.config]
+    if args.d:
+        import dataclasses
+        w = dataclasses.replace(w, d=args.d, name=f"{w.name}@d={args.d}")
     if args.impl == "reference":
         return run_reference(args, w)
 

@@ -8,7 +8,6 @@
 
 namespace aspis {
 
-size_t aggregate_smem_bytes(int64_t f, int *tc_out);
 
 int sm_count()
 {
@@ -123,8 +122,6 @@ extern "C" aspis_status aspis_aggregate(const float *copies, int64_t d, int64_t 
     if ((s = check_copies(copies, d, ld, a)) != ASPIS_OK) return s;
     if (!sel || !det || !out || (mode != 0 && mode != 1)) return ASPIS_E_INVAL;
     if (a->f > ASPIS_MAX_AGG_FILES) return ASPIS_E_RANGE;
-    int tc = 0;
-    if (!aggregate_smem_bytes(a->f, &tc) || !tc) return ASPIS_E_RANGE;
     return cuda_status(launch_aggregate(copies, a->f, a->r, d, ld, sel, det, mode, out,
                                         (cudaStream_t)stream));
 }

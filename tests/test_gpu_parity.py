@@ -317,3 +317,66 @@ def test_generator_torch_cuda_matches_numpy():
     host = synth.build_copies_np(w, oa.file_workers)
     dev = synth.build_copies_torch(w, oa.file_workers, DEV)
     assert np.array_equal(dev.cpu().numpy().view(np.uint32), host.view(np.uint32))
+
+
+# ------------------------------------------------ exact fallback paths of the median
+
+
+def _median_case(vals):
+    """vals: float32 [n, d] chosen values; run aggregate with one copy per
+    file (r=2, both copies equal) so that every file is kept as is."""
+    n, d = vals.shape
+    K = next(k for k in range(2, 200) if math.comb(k, 2) >= n)
+    f = math.comb(K, 2)
+    host = np.zeros((f, 2, d), np.float32)
+    rows = np.concatenate([vals, np.repeat(vals[-1:], f - n, axis=0)]) if f > n else vals
+    host[:, 0] = rows
+    host[:, 1] = rows
+    oa = oracle.assign(K, 2)
+    want = oracle.run_round(host, oa, d)
+    a = ap.aspis_assign(K, 2)
+    buf = gpu_round(ap, torch, torch.from_numpy(host).to(DEV), d, a)
+    assert_round_matches(ap, buf, want)
+
+
+def test_median_nan_inf_outside_sampled_rows():
+    rng = np.random.default_rng(12)
+    n, d = 455, 96
+    vals = rng.standard_normal((n, d)).astype(np.float32)
+    u = vals.view(np.uint32)
+    for c in range(d):
+        rows = rng.choice(np.arange(100, n), size=3, replace=False)
+        kind = c % 6
+        pat = [0xffc00000, 0x7fc00000, 0xff800000, 0x7f800000, 0xffc00123, 0x80000000][kind]
+        u[rows, c] = pat
+    _median_case(vals)
+
+
+def test_median_heavy_ties_overflow_bin():
+    rng = np.random.default_rng(13)
+    n, d = 455, 64
+    vals = rng.standard_normal((n, d)).astype(np.float32)
+    med = np.sort(vals, axis=0)[(n - 1) // 2]
+    for c in range(d):
+        rows = rng.choice(np.arange(64, n), size=60, replace=False)
+        vals[rows, c] = med[c]               # 60 ties straddle the median
+    _median_case(vals)
+
+
+def test_median_candidates_concentrated_in_one_lane():
+    rng = np.random.default_rng(14)
+    n, d = 455, 64
+    vals = rng.standard_normal((n, d)).astype(np.float32)
+    for c in range(d):
+        med = float(np.sort(vals[:, c])[(n - 1) // 2])
+        rows = np.arange(64, n, 8)[:20]      # one row group: one lane holds them all
+        vals[rows, c] = (med + np.arange(20) * 1e-6).astype(np.float32)
+    _median_case(vals)
+
+
+def test_median_wide_range_and_subnormals():
+    rng = np.random.default_rng(15)
+    n, d = 300, 64
+    mag = 10.0 ** rng.uniform(-44, 38, (n, d))
+    vals = (rng.choice([-1.0, 1.0], (n, d)) * mag).astype(np.float32)
+    _median_case(vals)
