@@ -3,8 +3,8 @@
 //
 // Data path.  Persistent CTAs of 8 warps.  A tile is TC consecutive
 // coordinates of all n kept rows.  It is staged in shared memory by 16-byte
-// cp.async copies in which 8 consecutive lanes fetch one row's 128 bytes, so
-// every memory request carries a whole line (a gather of 16-byte pieces of
+// cp.async copies in which consecutive lanes fetch one row's 16*TC/4 bytes,
+// so every memory request carries whole lines (a gather of 16-byte pieces of
 // many rows runs ~10x below the streaming rate).  Either two CTAs share an SM
 // with one tile each (their load and reduce phases overlap), or one CTA
 // keeps STAGES tiles in flight.  Rows of a tile are TC floats; the 16-byte
@@ -22,22 +22,23 @@
 // Lower median, exact (IEEE totalOrder through a monotone uint32 key; the
 // key map is a bijection, so the output has the chosen element's bits).  Per
 // coordinate, a small state machine:
-//   VH  value-space histogram: 256 bins, bins 1..254 evenly over the range of
-//       a sample (each lane's first value), 0 / 255 catching everything below
-//       / above.  The bin map x -> bits(fma(x, s, c)) - bits(2^23), clamped,
-//       is monotone in totalOrder, so bins are contiguous value ranges; a
-//       scan over the coordinate's lanes finds the bin holding the target
-//       rank.  (Key-space bins cannot do this in one pass: values of both
-//       signs near zero span ~2^31 keys.)
-//   VC  each lane copies the keys of that bin (at most kSlots per lane) and
+//   VH  value-space histogram: 128 bins, bins 1..126 evenly over the range of
+//       a sample (two values per lane), 0 / 127 catching everything below /
+//       above.  The bin map x -> bits(fma(x, s, c)) - bits(2^23), clamped,
+//       is monotone in totalOrder, so bins are contiguous value ranges; each
+//       value's bin is also kept as a byte.  A scan over the coordinate's
+//       lanes finds the bin holding the target rank.  (Key-space bins cannot
+//       do this in one pass: values of both signs near zero span ~2^31 keys.)
+//   VC  each lane compares its bytes with that bin (branch-free, 32 rows at
+//       a time into a bit mask; rows past n hold a byte no bin has), the
+//       members' keys are stored at a prefix over the coordinate's lanes and
 //       the <= 32 of them are ranked directly.
 // Exact fallback, taken when the sample range is degenerate or not finite,
-// a NaN is seen, the bin holds more than 32 values or a lane runs out of
-// slots:
+// a NaN is seen or the bin holds more than 32 values:
 //   KA  min / max of the keys -> range [lo, hi]
-//   KH  256 equal-width key-space bins over [lo, hi]; the bin holding the
-//       rank becomes [lo, hi] (each pass shrinks the range by at least 2^7)
-//   KC  as VC for the keys left in [lo, hi].
+//   KH  128 equal-width key-space bins over [lo, hi]; the bin holding the
+//       rank becomes [lo, hi] (each pass shrinks the range by at least 2^6)
+//   KC  the keys left in [lo, hi] are gathered with warp ballots and ranked.
 // The pass cap only guards against an inconsistent state.
 #include <climits>
 
@@ -48,12 +49,11 @@ namespace {
 
 constexpr int kThreads = 256;     // 8 warps
 constexpr int kWarps = kThreads / 32;
-constexpr int kNB = 256;          // histogram bins per pass
-constexpr int kLogNB = 8;
+constexpr int kNB = 128;          // histogram bins per pass
+constexpr int kLogNB = 7;
 constexpr int kHistStride = kNB + 4;   // words per coordinate row (rows start 4 banks apart)
 constexpr int kCap = 32;          // keys ranked directly
-constexpr int kSlots = 8;         // candidate slots per lane
-constexpr int kSlotStride = kSlots + 1;
+constexpr int kListStride = kCap + 1;
 
 __device__ __forceinline__ uint32_t to_key(uint32_t u)
 {
@@ -92,16 +92,14 @@ __device__ __forceinline__ void col_sync(int cw)
 }
 
 // Value-space bin of y = fma(x, s, c): the integer part of y read from its
-// bits (y is near 2^23, where one unit is one ulp), clamped to [0, 255].
-// Rounding is monotone and the clamp sends negative y, -inf and -NaN-free
-// underflow to 0 and +inf / large y to 255, so the map is monotone in the
-// IEEE totalOrder of x for every non-NaN x (NaNs are detected separately:
-// fma returns a canonical NaN whatever the sign of x).
-__device__ __forceinline__ int vraw(float y) { return (int)__float_as_uint(y) - 0x4B000000; }
-
+// bits (y is near 2^23, where one unit is one ulp), clamped to [0, kNB).
+// Rounding is monotone and the clamp sends negative y, -inf and underflow
+// to 0 and +inf / large y to kNB-1, so the map is monotone in the IEEE
+// totalOrder of x for every non-NaN x.  NaNs are detected separately: fma
+// returns a canonical NaN whatever the sign of x.
 __device__ __forceinline__ uint32_t vbin(float y)
 {
-    return (uint32_t)min(max(vraw(y), 0), kNB - 1);
+    return (uint32_t)min(max((int)__float_as_uint(y) - 0x4B000000, 0), kNB - 1);
 }
 
 enum { M_DONE = 0, M_VH, M_VC, M_KA, M_KH, M_KC };
@@ -115,22 +113,26 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e)
 }
 
 struct Layout {
-    size_t tiles, rows, hist, cand, ccnt, red, state, total, tile_bytes;
+    size_t tiles, bins, rows, hist, list, lcnt, red, state, total, tile_bytes;
 };
+
+template <int TC>
+__host__ __device__ constexpr int bin_pitch() { return TC + 4; }   // bytes per row of bins
 
 template <int TC, int STAGES>
 __host__ __device__ inline Layout make_layout(int64_t f)
 {
-    constexpr int G = 8 * (kWarps / (TC / 4));
+    constexpr int WS = kWarps / (TC / 4);
     Layout L{};
     size_t o = 0;
     L.tile_bytes = ((size_t)f * TC * 4 + 127) / 128 * 128;
     L.tiles = o; o += STAGES * L.tile_bytes;
+    L.bins = o; o += ((size_t)(f + 32 * 8 * WS) * bin_pitch<TC>() + 15) / 16 * 16;
     L.rows = o; o += ((size_t)f * 4 + 15) / 16 * 16;
     L.hist = o; o += (size_t)TC * kHistStride * 4;
-    L.cand = o; o += (size_t)TC * G * kSlotStride * 4;
-    L.ccnt = o; o += (size_t)TC * G * 4;
-    L.red = o; o += (size_t)TC * G * 8;
+    L.list = o; o += (size_t)TC * WS * kListStride * 4;
+    L.lcnt = o; o += (size_t)TC * WS * 4;
+    L.red = o; o += (size_t)TC * WS * 8;
     L.state = o; o += (size_t)TC * 8 * 4;
     L.total = o;
     return L;
@@ -145,16 +147,18 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     constexpr int WS = kWarps / CPR;       // warps per chunk column
     constexpr int G = 8 * WS;              // lanes per coordinate
     constexpr int RPL = 32 / TC;           // tile rows per 128-byte line
-    constexpr int BPL = kNB / G;           // histogram bins summed per lane
+    constexpr int BPL = kNB / G;           // histogram bins summed per lane (16, 8, 4, 2)
     constexpr int RPI = kThreads / CPR;    // tile rows covered by one copy round
+    constexpr int BP = bin_pitch<TC>();
     extern __shared__ __align__(128) unsigned char smem[];
     const Layout L = make_layout<TC, STAGES>(f);
     unsigned char *tiles = smem + L.tiles;
+    uint8_t *bins = smem + L.bins;                                    // [n][BP] bytes
     int32_t *rows = reinterpret_cast<int32_t *>(smem + L.rows);
     uint32_t *hist = reinterpret_cast<uint32_t *>(smem + L.hist);     // [TC][kHistStride]
-    uint32_t *cand = reinterpret_cast<uint32_t *>(smem + L.cand);     // [TC][G][kSlotStride]
-    uint32_t *ccnt = reinterpret_cast<uint32_t *>(smem + L.ccnt);     // [TC][G]
-    uint32_t *red = reinterpret_cast<uint32_t *>(smem + L.red);       // [TC][G][2]
+    uint32_t *list = reinterpret_cast<uint32_t *>(smem + L.list);     // [TC][WS][kListStride]
+    uint32_t *lcnt = reinterpret_cast<uint32_t *>(smem + L.lcnt);     // [TC][WS]
+    uint32_t *red = reinterpret_cast<uint32_t *>(smem + L.red);       // [TC][WS][2]
     uint32_t *st = reinterpret_cast<uint32_t *>(smem + L.state);      // [8][TC]
     __shared__ int warp_tot[kWarps];
 
@@ -190,11 +194,14 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     }
     const uint32_t krank = (uint32_t)((n - 1) / 2);
     const int64_t ntiles = (d + TC - 1) / TC;
+    // rows past n read as bin 0xFF, which no value has (bins are < kNB)
+    for (int e = tid; e < 32 * G * BP; e += kThreads) bins[n * BP + e] = 0xFFu;
 
     // lane's first element (in words) and the stride between its rows
     const int fl = (gf / RPL) & (CPR - 1);
     const int off0 = gf * TC + ((cw ^ fl) << 2) + cq;
     constexpr int kStride = G * TC;
+    constexpr int kBStride = G * BP;
     const int nmine = n > gf ? (n - gf + G - 1) / G : 0;
 
     // copy role (vector path): this thread always moves chunk ch_me of rows
@@ -264,26 +271,34 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             }
             if constexpr (WS > 1) {
                 if (g8 == 0) {
-                    red[(cc * G + ws) * 2] = __float_as_uint(s);
-                    red[(cc * G + ws) * 2 + 1] = __float_as_uint(e);
+                    red[(cc * WS + ws) * 2] = __float_as_uint(s);
+                    red[(cc * WS + ws) * 2 + 1] = __float_as_uint(e);
                 }
                 col_sync<WS>(cw);
                 s = 0.f;
                 e = 0.f;
                 for (int u = 0; u < WS; ++u) {
                     float ns, ne;
-                    two_sum(s, __uint_as_float(red[(cc * G + u) * 2]), ns, ne);
+                    two_sum(s, __uint_as_float(red[(cc * WS + u) * 2]), ns, ne);
                     s = ns;
-                    e += ne + __uint_as_float(red[(cc * G + u) * 2 + 1]);
+                    e += ne + __uint_as_float(red[(cc * WS + u) * 2 + 1]);
                 }
             }
             if (gf == 0 && live) out[c0 + cc] = (float)(((double)s + (double)e) / (double)n);
         } else {
-            // ---- sample range: the first value of each lane of the coordinate.
-            // Value-space bins 1..254 split [sample min, sample max] evenly;
-            // bins 0 and 255 catch everything below / above (see vbin below).
-            uint32_t slo = nmine > 0 ? to_key(tile[off0]) : 0xffffffffu;
-            uint32_t shi = nmine > 0 ? slo : 0u;
+            // ---- sample range: the first two values of each lane of the
+            // coordinate; bins 1..kNB-2 split [min, max] of the sample evenly
+            uint32_t slo = 0xffffffffu, shi = 0u;
+            if (nmine > 0) {
+                const uint32_t k = to_key(tile[off0]);
+                slo = min(slo, k);
+                shi = max(shi, k);
+            }
+            if (nmine > 1) {
+                const uint32_t k = to_key(tile[off0 + kStride]);
+                slo = min(slo, k);
+                shi = max(shi, k);
+            }
 #pragma unroll
             for (int o = 4; o < 32; o <<= 1) {
                 slo = min(slo, __shfl_xor_sync(full, slo, o));
@@ -291,32 +306,33 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             }
             if constexpr (WS > 1) {
                 if (g8 == 0) {
-                    red[(cc * G + ws) * 2] = slo;
-                    red[(cc * G + ws) * 2 + 1] = shi;
+                    red[(cc * WS + ws) * 2] = slo;
+                    red[(cc * WS + ws) * 2 + 1] = shi;
                 }
                 if (gf == 0) st[4 * TC + cc] = 0u;     // NaN flag of this tile
                 col_sync<WS>(cw);
                 for (int u = 0; u < WS; ++u) {
-                    slo = min(slo, red[(cc * G + u) * 2]);
-                    shi = max(shi, red[(cc * G + u) * 2 + 1]);
+                    slo = min(slo, red[(cc * WS + u) * 2]);
+                    shi = max(shi, red[(cc * WS + u) * 2 + 1]);
                 }
                 col_sync<WS>(cw);
             }
             const float xs_lo = __uint_as_float(from_key(slo));
             const float xs_hi = __uint_as_float(from_key(shi));
-            const float vs = 254.0f / (xs_hi - xs_lo);
+            const float vs = (float)(kNB - 2) / (xs_hi - xs_lo);
             const float vc = 8388609.0f - xs_lo * vs;    // xs_lo -> about 2^23 + 1
             const bool vspace = isfinite(xs_lo) && isfinite(xs_hi) && xs_hi > xs_lo &&
                                 isfinite(vs) && isfinite(vc);
 
             int mode = !live ? M_DONE : (vspace ? M_VH : M_KA);
-            uint32_t lo = 0u, hi = 0u, krem = krank, cnt = (uint32_t)n, res = 0u;
-            int vlo = 0, vhi = 0;           // raw value-space bin bounds of the chosen bin
+            uint32_t lo = 0u, hi = 0u, krem = krank, cnt = (uint32_t)n, res = 0u, vb = 0u;
+            uint8_t *bmine = bins + gf * BP + cc;       // this lane's first bin byte
 
             for (int pass = 0; pass < 20; ++pass) {
                 // the column's warps hold identical states: the exit is uniform
                 if ((__ballot_sync(full, mode == M_DONE) & 0xfu) == 0xfu) break;
                 const int m0 = mode;
+                const bool cmode = m0 == M_VC || m0 == M_KC;
                 const uint32_t W = hi - lo;
                 const int bits = 32 - __clz(W);
                 const int sh = bits > kLogNB ? bits - kLogNB : 0;
@@ -328,37 +344,34 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
 
                 // ---- sweep over the lane's values
                 const uint32_t *p = tile + off0;
-                uint32_t mycnt = 0, amin = 0xffffffffu, amax = 0u;
+                uint32_t amin = 0xffffffffu, amax = 0u;
                 bool nanf = false;
-                uint32_t *slots = cand + (cc * G + gf) * kSlotStride;
                 if (m0 == M_VH) {
+                    uint8_t *pb = bmine;
                     int j = 0;
-                    for (; j + 4 <= nmine; j += 4, p += 4 * kStride) {
+                    for (; j + 4 <= nmine; j += 4, p += 4 * kStride, pb += 4 * kBStride) {
                         const float y0 = fmaf(__uint_as_float(p[0]), vs, vc);
                         const float y1 = fmaf(__uint_as_float(p[kStride]), vs, vc);
                         const float y2 = fmaf(__uint_as_float(p[2 * kStride]), vs, vc);
                         const float y3 = fmaf(__uint_as_float(p[3 * kStride]), vs, vc);
                         nanf |= (y0 != y0) | (y1 != y1) | (y2 != y2) | (y3 != y3);
-                        atomicAdd(h + vbin(y0), 1u);
-                        atomicAdd(h + vbin(y1), 1u);
-                        atomicAdd(h + vbin(y2), 1u);
-                        atomicAdd(h + vbin(y3), 1u);
+                        const uint32_t b0 = vbin(y0), b1 = vbin(y1), b2 = vbin(y2), b3 = vbin(y3);
+                        atomicAdd(h + b0, 1u);
+                        atomicAdd(h + b1, 1u);
+                        atomicAdd(h + b2, 1u);
+                        atomicAdd(h + b3, 1u);
+                        pb[0] = (uint8_t)b0;
+                        pb[kBStride] = (uint8_t)b1;
+                        pb[2 * kBStride] = (uint8_t)b2;
+                        pb[3 * kBStride] = (uint8_t)b3;
                     }
-                    for (; j < nmine; ++j, p += kStride) {
+                    for (; j < nmine; ++j, p += kStride, pb += kBStride) {
                         const float y = fmaf(__uint_as_float(*p), vs, vc);
                         nanf |= y != y;
-                        atomicAdd(h + vbin(y), 1u);
+                        const uint32_t b = vbin(y);
+                        atomicAdd(h + b, 1u);
+                        *pb = (uint8_t)b;
                     }
-                } else if (m0 == M_VC) {
-                    for (int j = 0; j < nmine; ++j, p += kStride) {
-                        const uint32_t u = *p;
-                        const int raw = vraw(fmaf(__uint_as_float(u), vs, vc));
-                        if (raw >= vlo && raw <= vhi) {
-                            if (mycnt < (uint32_t)kSlots) slots[mycnt] = to_key(u);
-                            ++mycnt;
-                        }
-                    }
-                    ccnt[cc * G + gf] = mycnt;
                 } else if (m0 == M_KA) {
                     for (int j = 0; j < nmine; ++j, p += kStride) {
                         const uint32_t k = to_key(*p);
@@ -370,15 +383,53 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                         const uint32_t dk = to_key(*p) - lo;
                         if (dk <= W) atomicAdd(h + (dk >> sh), 1u);
                     }
-                } else if (m0 == M_KC) {
-                    for (int j = 0; j < nmine; ++j, p += kStride) {
-                        const uint32_t k = to_key(*p);
-                        if (k - lo <= W) {
-                            if (mycnt < (uint32_t)kSlots) slots[mycnt] = k;
-                            ++mycnt;
+                }
+                // VC: byte compare into per-lane masks of 32 rows, then the
+                // members are stored at a prefix over the coordinate's lanes
+                if (__any_sync(full, m0 == M_VC)) {
+                    uint32_t *lst = list + (cc * WS + ws) * kListStride;
+                    const int iters = (int)__reduce_max_sync(full, m0 == M_VC ? (unsigned)nmine : 0u);
+                    uint32_t nlist = 0u;
+                    for (int jb = 0; jb < iters; jb += 32) {
+                        const uint8_t *pb = bmine + jb * kBStride;
+                        uint32_t mask = 0u;
+#pragma unroll
+                        for (int jj = 0; jj < 32; ++jj)
+                            mask |= (pb[jj * kBStride] == vb ? 1u : 0u) << jj;
+                        if (m0 != M_VC) mask = 0u;
+                        const uint32_t cntm = __popc(mask);
+                        uint32_t incl = cntm;
+#pragma unroll
+                        for (int o = 1; o < 8; o <<= 1) {
+                            const uint32_t tv = __shfl_up_sync(full, incl, 4 * o);
+                            if (g8 >= o) incl += tv;
+                        }
+                        const uint32_t tot = __shfl_sync(full, incl, 28 + cq);
+                        uint32_t pos = nlist + incl - cntm;
+                        while (mask) {
+                            const int jj = __ffs(mask) - 1;
+                            mask &= mask - 1;
+                            lst[pos++] = to_key(tile[off0 + (jb + jj) * kStride]);
+                        }
+                        nlist += tot;
+                    }
+                    if (m0 == M_VC && g8 == 0) lcnt[cc * WS + ws] = nlist;
+                }
+                // KC (fallback): ballot-gathered list of the keys in [lo, hi]
+                if (__any_sync(full, m0 == M_KC)) {
+                    uint32_t *lst = list + (cc * WS + ws) * kListStride;
+                    const int iters = (int)__reduce_max_sync(full, m0 == M_KC ? (unsigned)nmine : 0u);
+                    const uint32_t *pc = tile + off0;
+                    uint32_t nlist = 0u;
+                    for (int j = 0; j < iters; ++j, pc += kStride) {
+                        const bool pk = m0 == M_KC && j < nmine && to_key(*pc) - lo <= W;
+                        const unsigned m = __ballot_sync(full, pk);
+                        if (m) {
+                            if (pk) lst[nlist + __popc(m & seg & below)] = to_key(*pc);
+                            nlist += __popc(m & seg);
                         }
                     }
-                    ccnt[cc * G + gf] = mycnt;
+                    if (m0 == M_KC && g8 == 0) lcnt[cc * WS + ws] = nlist;
                 }
                 bool nan_any = false;
                 if constexpr (WS == 1) {
@@ -389,7 +440,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 col_sync<WS>(cw);
                 if constexpr (WS > 1) nan_any = st[4 * TC + cc] != 0u;
 
-                // ---- key range of the fallback path (pass A)
+                // ---- key range of the fallback path (pass KA)
                 if (__any_sync(full, m0 == M_KA)) {
 #pragma unroll
                     for (int o = 4; o < 32; o <<= 1) {
@@ -398,13 +449,13 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     }
                     if constexpr (WS > 1) {
                         if (g8 == 0) {
-                            red[(cc * G + ws) * 2] = amin;
-                            red[(cc * G + ws) * 2 + 1] = amax;
+                            red[(cc * WS + ws) * 2] = amin;
+                            red[(cc * WS + ws) * 2 + 1] = amax;
                         }
                         col_sync<WS>(cw);
                         for (int u = 0; u < WS; ++u) {
-                            amin = min(amin, red[(cc * G + u) * 2]);
-                            amax = max(amax, red[(cc * G + u) * 2 + 1]);
+                            amin = min(amin, red[(cc * WS + u) * 2]);
+                            amax = max(amax, red[(cc * WS + u) * 2 + 1]);
                         }
                         col_sync<WS>(cw);
                     }
@@ -427,7 +478,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 uint32_t nbin = 0, nrr = 0, ncb = 0;
                 if constexpr (WS == 1) {
                     if (__any_sync(full, hm)) {
-                        // level 1: lane g8 sums bins [32*g8, 32*g8 + 32); scan over g8
+                        // level 1: lane g8 sums bins [16*g8, 16*g8 + 16); scan over g8
                         uint32_t sum = 0;
 #pragma unroll
                         for (int b = 0; b < BPL; b += 4) {
@@ -444,9 +495,9 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                         const int owner = m1 ? __ffs(m1) - 1 : cq;
                         const uint32_t before = __shfl_sync(full, incl - sum, owner);
                         const int og = owner >> 2;
-                        // level 2: lane g8 takes 4 bins of the owner's 32
-                        const uint4 c = *reinterpret_cast<const uint4 *>(h + og * BPL + g8 * 4);
-                        const uint32_t s2 = (c.x + c.y) + (c.z + c.w);
+                        // level 2: lane g8 takes 2 bins of the owner's 16
+                        const uint2 c = *reinterpret_cast<const uint2 *>(h + og * BPL + g8 * 2);
+                        const uint32_t s2 = c.x + c.y;
                         uint32_t incl2 = s2;
 #pragma unroll
                         for (int o = 1; o < 8; o <<= 1) {
@@ -456,37 +507,28 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                         const uint32_t r2 = krem - before;
                         const unsigned m2 = __ballot_sync(full, incl2 > r2) & seg;
                         const int owner2 = m2 ? __ffs(m2) - 1 : cq;
-                        uint32_t rr = r2 - (incl2 - s2), cb = c.w;
-                        int b = 3;
+                        uint32_t rr = r2 - (incl2 - s2), cb = c.y;
+                        int b = 1;
                         if (rr < c.x) {
                             b = 0;
                             cb = c.x;
-                        } else if ((rr -= c.x) < c.y) {
-                            b = 1;
-                            cb = c.y;
-                        } else if ((rr -= c.y) < c.z) {
-                            b = 2;
-                            cb = c.z;
                         } else {
-                            rr -= c.z;
+                            rr -= c.x;
                         }
-                        const uint32_t bin = (uint32_t)(og * BPL + g8 * 4 + b);
+                        const uint32_t bin = (uint32_t)(og * BPL + g8 * 2 + b);
                         nbin = __shfl_sync(full, bin, owner2);
                         nrr = __shfl_sync(full, rr, owner2);
                         ncb = __shfl_sync(full, cb, owner2);
                     }
                 } else {
                     // WS warps per coordinate: per-lane partial sums through shared
-                    // memory (the coordinate's candidate slots are free here),
-                    // then the lane with gf == 0 finishes the search
-                    uint32_t *part = cand + cc * G * kSlotStride;
+                    // memory (the coordinate's list area is free here), then the
+                    // lane with gf == 0 finishes the search
+                    uint32_t *part = list + cc * WS * kListStride;    // G <= WS * kListStride
                     if (hm) {
                         uint32_t sum = 0;
 #pragma unroll
-                        for (int b = 0; b < BPL; b += 4) {
-                            const uint4 v = *reinterpret_cast<const uint4 *>(h + gf * BPL + b);
-                            sum += (v.x + v.y) + (v.z + v.w);
-                        }
+                        for (int b = 0; b < BPL; ++b) sum += h[gf * BPL + b];
                         part[gf] = sum;
                     }
                     col_sync<WS>(cw);
@@ -515,8 +557,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     if (nan_any || ncb > (uint32_t)kCap) {
                         mode = M_KA;             // exact key-space passes instead
                     } else {
-                        vlo = nbin == 0 ? INT_MIN : (int)nbin;
-                        vhi = nbin == kNB - 1 ? INT_MAX : (int)nbin;
+                        vb = nbin;
                         krem = nrr;
                         cnt = ncb;
                         mode = M_VC;
@@ -536,57 +577,63 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     }
                 }
 
-                // ---- ranking of the collected keys: every lane ranks its own
-                // candidates (two at a time) against all of the coordinate's
-                const bool cm = m0 == M_VC || m0 == M_KC;
-                bool ovf = false, any = false;
+                // ---- rank the listed keys: lane gf takes entries gf, gf+G, ...
+                bool any = false;
                 uint32_t hit = 0u;
-                if (cm) {
-                    for (int u = 0; u < G; ++u) ovf |= ccnt[cc * G + u] > (uint32_t)kSlots;
-                    if (!ovf) {
-                        const uint32_t mine = mycnt;
-                        for (uint32_t k0 = 0; k0 < mine; k0 += 2) {
-                            const uint32_t x0 = slots[k0];
-                            const bool two = k0 + 1 < mine;
-                            const uint32_t x1 = two ? slots[k0 + 1] : 0u;
-                            uint32_t lt0 = 0, le0 = 0, lt1 = 0, le1 = 0;
-                            for (int u = 0; u < G; ++u) {
-                                const uint32_t cu = ccnt[cc * G + u];
-                                const uint32_t *cl = cand + (cc * G + u) * kSlotStride;
-                                for (uint32_t t2 = 0; t2 < cu; ++t2) {
-                                    const uint32_t y = cl[t2];
-                                    lt0 += y < x0;
-                                    le0 += y <= x0;
-                                    lt1 += y < x1;
-                                    le1 += y <= x1;
-                                }
+                if constexpr (WS == 1) {
+                    if (__any_sync(full, cmode)) {
+                        const uint32_t cmax = __reduce_max_sync(full, cmode ? cnt : 0u);
+                        const uint32_t *cl = list + cc * kListStride;
+                        for (uint32_t e0 = (uint32_t)g8; e0 < cmax; e0 += 8) {
+                            const bool mine = cmode && e0 < cnt;
+                            const uint32_t x = mine ? cl[e0] : 0u;
+                            uint32_t lt = 0, le = 0;
+                            for (uint32_t t2 = 0; t2 < cmax; ++t2) {
+                                const uint32_t y = t2 < cnt ? cl[t2] : 0xffffffffu;
+                                lt += (t2 < cnt) & (y < x);
+                                le += (t2 < cnt) & (y <= x);
                             }
-                            if (lt0 <= krem && krem < le0) {
-                                hit = x0;
+                            if (mine && lt <= krem && krem < le) {
+                                hit = x;
                                 any = true;
                             }
-                            if (two && lt1 <= krem && krem < le1) {
-                                hit = x1;
-                                any = true;
+                        }
+                    }
+                } else if (cmode) {
+                    for (uint32_t e0 = (uint32_t)gf; e0 < cnt; e0 += G) {
+                        // entry e0 of the concatenated per-warp lists
+                        uint32_t m = e0;
+                        int u = 0;
+                        for (; u < WS - 1 && m >= lcnt[cc * WS + u]; ++u) m -= lcnt[cc * WS + u];
+                        const uint32_t x = list[(cc * WS + u) * kListStride + m];
+                        uint32_t lt = 0, le = 0;
+                        for (int u2 = 0; u2 < WS; ++u2) {
+                            const uint32_t cu = lcnt[cc * WS + u2];
+                            const uint32_t *cl = list + (cc * WS + u2) * kListStride;
+                            for (uint32_t t2 = 0; t2 < cu; ++t2) {
+                                const uint32_t y = cl[t2];
+                                lt += y < x;
+                                le += y <= x;
                             }
+                        }
+                        if (lt <= krem && krem < le) {
+                            hit = x;
+                            any = true;
                         }
                     }
                 }
                 if constexpr (WS == 1) {
                     const unsigned mh = __ballot_sync(full, any) & seg;
                     const uint32_t v = __shfl_sync(full, hit, mh ? __ffs(mh) - 1 : lane);
-                    if (cm && !ovf) res = v;
+                    if (cmode) res = v;
                 } else {
                     if (any) st[3 * TC + cc] = hit;
                     col_sync<WS>(cw);
-                    if (cm && !ovf) res = st[3 * TC + cc];
+                    if (cmode) res = st[3 * TC + cc];
                     if (gf == 0) st[4 * TC + cc] = 0u;   // NaN flag, next pass
                     col_sync<WS>(cw);
                 }
-                if (cm) {
-                    if (!ovf) mode = M_DONE;
-                    else mode = m0 == M_VC ? M_KA : M_KH;   // a lane ran out of slots
-                }
+                if (cmode) mode = M_DONE;
             }
             if (gf == 0 && live) out[c0 + cc] = __uint_as_float(from_key(res));
         }
@@ -645,8 +692,10 @@ cudaError_t launch_mode(const float *copies, int64_t f, int r, int64_t d, int64_
         ASPIS_TRY(16, 2, 1)
         ASPIS_TRY(8, 3, 1)
         ASPIS_TRY(8, 2, 1)
+        ASPIS_TRY(8, 1, 1)
+        ASPIS_TRY(4, 2, 1)
     }
-    ASPIS_TRY(4, 2, 1)
+    ASPIS_TRY(4, 1, 1)
 #undef ASPIS_TRY
     return cudaErrorInvalidValue;
 }
