@@ -218,7 +218,16 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 if (c < d) {
                     const float *src = copies + c;
                     uint32_t dst = sbase + (uint32_t)(i0_me * TC + sw_me * 4) * 4u;
-                    for (int i = i0_me; i < n; i += RPI, dst += RPI * TC * 4)
+                    int i = i0_me;
+                    for (; i + 3 * RPI < n; i += 4 * RPI, dst += 4 * RPI * TC * 4) {
+                        const int32_t r0 = rows[i], r1 = rows[i + RPI];
+                        const int32_t r2 = rows[i + 2 * RPI], r3 = rows[i + 3 * RPI];
+                        cp_async16(dst, src + (int64_t)r0 * ld);
+                        cp_async16(dst + RPI * TC * 4, src + (int64_t)r1 * ld);
+                        cp_async16(dst + 2 * RPI * TC * 4, src + (int64_t)r2 * ld);
+                        cp_async16(dst + 3 * RPI * TC * 4, src + (int64_t)r3 * ld);
+                    }
+                    for (; i < n; i += RPI, dst += RPI * TC * 4)
                         cp_async16(dst, src + (int64_t)rows[i] * ld);
                 }
             } else {
