@@ -265,6 +265,7 @@ def main():
         if ev:
             ev[3].record(stream)
 
+    stream.wait_stream(torch.cuda.current_stream())   # inputs were made on the default stream
     with torch.cuda.stream(stream):
         for _ in range(max(3, args.warmup)):
             one_round()
