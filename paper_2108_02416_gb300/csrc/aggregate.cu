@@ -33,37 +33,33 @@
 //       a time into a bit mask; rows past n hold a byte no bin has), the
 //       members' keys are stored at a prefix over the coordinate's lanes and
 //       the <= 32 of them are ranked directly.
-// Exact fallback, taken when the sample range is degenerate or not finite,
-// a NaN is seen or the bin holds more than 32 values:
+//   VM  a bin with more than 32 members: their exact key range [lo, hi];
+//   VR  value-space bins over that range for the members only (every other
+//       tag becomes 0xFF), then VC or VM again.  At most two such levels,
+//       each at least 4x smaller; otherwise key-space passes on [lo, hi].
+// Exact key-space fallback, taken when the sample range is degenerate or not
+// finite, a NaN is seen or refinement stalls:
 //   KA  min / max of the keys -> range [lo, hi]
 //   KH  128 equal-width key-space bins over [lo, hi]; the bin holding the
 //       rank becomes [lo, hi] (each pass shrinks the range by at least 2^6)
 //   KC  the keys left in [lo, hi] are gathered with warp ballots and ranked.
-// The pass cap only guards against an inconsistent state.
+// One pass body serves every mode; it is instantiated three times: a VH-only
+// pass and a VC-only pass that every tile runs first (the common case ends
+// there), and the general pass, looped only while a coordinate is left.  The
+// pass cap only guards against an inconsistent state.
 #include <climits>
+#include <type_traits>
 
 #include "aspis_internal.cuh"
+#include "median_common.cuh"
 
 namespace aspis {
 namespace {
 
 constexpr int kThreads = 256;     // 8 warps
 constexpr int kWarps = kThreads / 32;
-constexpr int kNB = 128;          // histogram bins per pass
-constexpr int kLogNB = 7;
 constexpr int kHistStride = kNB + 4;   // words per coordinate row (rows start 4 banks apart)
-constexpr int kCap = 32;          // keys ranked directly
 constexpr int kListStride = kCap + 1;
-
-__device__ __forceinline__ uint32_t to_key(uint32_t u)
-{
-    return u ^ ((uint32_t)((int32_t)u >> 31) | 0x80000000u);
-}
-
-__device__ __forceinline__ uint32_t from_key(uint32_t k)
-{
-    return k ^ ((uint32_t)((int32_t)~k >> 31) | 0x80000000u);
-}
 
 __device__ __forceinline__ void cp_async16(uint32_t saddr, const void *g)
 {
@@ -89,27 +85,6 @@ __device__ __forceinline__ void col_sync(int cw)
     } else {
         asm volatile("bar.sync %0, %1;\n" ::"r"(cw + 1), "r"(WS * 32) : "memory");
     }
-}
-
-// Value-space bin of y = fma(x, s, c): the integer part of y read from its
-// bits (y is near 2^23, where one unit is one ulp), clamped to [0, kNB).
-// Rounding is monotone and the clamp sends negative y, -inf and underflow
-// to 0 and +inf / large y to kNB-1, so the map is monotone in the IEEE
-// totalOrder of x for every non-NaN x.  NaNs are detected separately: fma
-// returns a canonical NaN whatever the sign of x.
-__device__ __forceinline__ uint32_t vbin(float y)
-{
-    return (uint32_t)min(max((int)__float_as_uint(y) - 0x4B000000, 0), kNB - 1);
-}
-
-enum { M_DONE = 0, M_VH, M_VC, M_KA, M_KH, M_KC };
-
-// Two-sum: s + e == a + b exactly (Knuth); no products, so nothing to fuse.
-__device__ __forceinline__ void two_sum(float a, float b, float &s, float &e)
-{
-    s = a + b;
-    const float bp = s - a;
-    e = (a - (s - bp)) + (b - bp);
 }
 
 struct Layout {
@@ -330,23 +305,25 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             const float xs_hi = __uint_as_float(from_key(shi));
             const float vs = (float)(kNB - 2) / (xs_hi - xs_lo);
             const float vc = 8388609.0f - xs_lo * vs;    // xs_lo -> about 2^23 + 1
+            float rs = 0.f, rc = 0.f;                    // bin map of the refinement passes
             const bool vspace = isfinite(xs_lo) && isfinite(xs_hi) && xs_hi > xs_lo &&
                                 isfinite(vs) && isfinite(vc);
 
             int mode = !live ? M_DONE : (vspace ? M_VH : M_KA);
             uint32_t lo = 0u, hi = 0u, krem = krank, cnt = (uint32_t)n, res = 0u, vb = 0u;
+            int vr_levels = 0;
             uint8_t *bmine = bins + gf * BP + cc;       // this lane's first bin byte
 
-            for (int pass = 0; pass < 20; ++pass) {
-                // the column's warps hold identical states: the exit is uniform
-                if ((__ballot_sync(full, mode == M_DONE) & 0xfu) == 0xfu) break;
+            auto pass = [&](auto kind) {
+
+                constexpr int K = decltype(kind)::value;   // 0 all modes, 1 VH only, 2 VC only
                 const int m0 = mode;
                 const bool cmode = m0 == M_VC || m0 == M_KC;
                 const uint32_t W = hi - lo;
                 const int bits = 32 - __clz(W);
                 const int sh = bits > kLogNB ? bits - kLogNB : 0;
                 uint32_t *h = hist + cc * kHistStride;
-                if (m0 == M_VH || m0 == M_KH)
+                if (K != 2 && (m0 == M_VH || m0 == M_KH || m0 == M_VR))
                     for (int b = gf * 4; b < kNB; b += G * 4)
                         *reinterpret_cast<uint4 *>(h + b) = make_uint4(0u, 0u, 0u, 0u);
                 col_sync<WS>(cw);
@@ -355,7 +332,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 const uint32_t *p = tile + off0;
                 uint32_t amin = 0xffffffffu, amax = 0u;
                 bool nanf = false;
-                if (m0 == M_VH) {
+                if (K != 2 && m0 == M_VH) {
                     uint8_t *pb = bmine;
                     int j = 0;
                     for (; j + 4 <= nmine; j += 4, p += 4 * kStride, pb += 4 * kBStride) {
@@ -381,7 +358,9 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                         atomicAdd(h + b, 1u);
                         *pb = (uint8_t)b;
                     }
-                } else if (m0 == M_KA) {
+                }
+                if constexpr (K == 0) {
+                if (m0 == M_KA) {
                     for (int j = 0; j < nmine; ++j, p += kStride) {
                         const uint32_t k = to_key(*p);
                         amin = min(amin, k);
@@ -393,8 +372,10 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                         if (dk <= W) atomicAdd(h + (dk >> sh), 1u);
                     }
                 }
+                }
                 // VC: byte compare into per-lane masks of 32 rows, then the
                 // members are stored at a prefix over the coordinate's lanes
+                if constexpr (K != 1) {
                 if (__any_sync(full, m0 == M_VC)) {
                     uint32_t *lst = list + (cc * WS + ws) * kListStride;
                     const int iters = (int)__reduce_max_sync(full, m0 == M_VC ? (unsigned)nmine : 0u);
@@ -424,6 +405,66 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     }
                     if (m0 == M_VC && g8 == 0) lcnt[cc * WS + ws] = nlist;
                 }
+                }
+                if constexpr (K == 0) {
+                // VM: key range of the members of bin vb (too many to list)
+                if (__any_sync(full, m0 == M_VM)) {
+                    uint32_t kmin = 0xffffffffu, kmax = 0u;
+                    if (m0 == M_VM)
+                        for (int j = 0; j < nmine; ++j)
+                            if (bmine[j * kBStride] == vb) {
+                                const uint32_t k = to_key(tile[off0 + j * kStride]);
+                                kmin = min(kmin, k);
+                                kmax = max(kmax, k);
+                            }
+#pragma unroll
+                    for (int o = 4; o < 32; o <<= 1) {
+                        kmin = min(kmin, __shfl_xor_sync(full, kmin, o));
+                        kmax = max(kmax, __shfl_xor_sync(full, kmax, o));
+                    }
+                    if constexpr (WS > 1) {
+                        if (g8 == 0 && m0 == M_VM) {
+                            red[(cc * WS + ws) * 2] = kmin;
+                            red[(cc * WS + ws) * 2 + 1] = kmax;
+                        }
+                        col_sync<WS>(cw);
+                        if (m0 == M_VM)
+                            for (int u = 0; u < WS; ++u) {
+                                kmin = min(kmin, red[(cc * WS + u) * 2]);
+                                kmax = max(kmax, red[(cc * WS + u) * 2 + 1]);
+                            }
+                        col_sync<WS>(cw);
+                    }
+                    if (m0 == M_VM) {
+                        // members are the values with keys in [kmin, kmax]: bins are
+                        // contiguous value ranges at every level
+                        lo = kmin;
+                        hi = kmax;
+                        if (lo == hi) {
+                            res = lo;
+                            mode = M_DONE;
+                        } else {
+                            const float xlo = __uint_as_float(from_key(kmin));
+                            const float xhi = __uint_as_float(from_key(kmax));
+                            rs = (float)(kNB - 2) / (xhi - xlo);
+                            rc = 8388609.0f - xlo * rs;
+                            mode = isfinite(rs) && isfinite(rc) && rs > 0.f ? M_VR : M_KH;
+                        }
+                    }
+                }
+                // VR: value-space bins over [kmin, kmax] for the members only;
+                // every other tag becomes 0xFF, which no bin has
+                if (m0 == M_VR) {
+                    uint8_t *pbr = bmine;
+                    for (int j = 0; j < nmine; ++j, pbr += kBStride) {
+                        uint32_t b = 0xFFu;
+                        if (*pbr == vb) {
+                            b = vbin(fmaf(__uint_as_float(tile[off0 + j * kStride]), rs, rc));
+                            atomicAdd(h + b, 1u);
+                        }
+                        *pbr = (uint8_t)b;
+                    }
+                }
                 // KC (fallback): ballot-gathered list of the keys in [lo, hi]
                 if (__any_sync(full, m0 == M_KC)) {
                     uint32_t *lst = list + (cc * WS + ws) * kListStride;
@@ -440,6 +481,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     }
                     if (m0 == M_KC && g8 == 0) lcnt[cc * WS + ws] = nlist;
                 }
+                }
                 bool nan_any = false;
                 if constexpr (WS == 1) {
                     nan_any = (__ballot_sync(full, nanf) & seg) != 0u;
@@ -449,6 +491,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 col_sync<WS>(cw);
                 if constexpr (WS > 1) nan_any = st[4 * TC + cc] != 0u;
 
+                if constexpr (K == 0) {
                 // ---- key range of the fallback path (pass KA)
                 if (__any_sync(full, m0 == M_KA)) {
 #pragma unroll
@@ -482,9 +525,11 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     }
                 }
 
+                }
                 // ---- bin search (value-space or key-space histogram)
-                const bool hm = m0 == M_VH || m0 == M_KH;
+                const bool hm = m0 == M_VH || m0 == M_KH || m0 == M_VR;
                 uint32_t nbin = 0, nrr = 0, ncb = 0;
+                if constexpr (K != 2) {
                 if constexpr (WS == 1) {
                     if (__any_sync(full, hm)) {
                         // level 1: lane g8 sums bins [16*g8, 16*g8 + 16); scan over g8
@@ -562,16 +607,22 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     nrr = st[1 * TC + cc];
                     ncb = st[2 * TC + cc];
                 }
-                if (m0 == M_VH) {
-                    if (nan_any || ncb > (uint32_t)kCap) {
+                }
+                if (K != 2 && (m0 == M_VH || m0 == M_VR)) {
+                    if (nan_any) {
                         mode = M_KA;             // exact key-space passes instead
+                    } else if (m0 == M_VR && ncb > (uint32_t)kCap &&
+                               (4u * ncb > cnt || ++vr_levels >= 2)) {
+                        // little progress (values spread over many scales, say):
+                        // key-space bins on the members' range [lo, hi] instead
+                        mode = M_KH;
                     } else {
                         vb = nbin;
                         krem = nrr;
                         cnt = ncb;
-                        mode = M_VC;
+                        mode = ncb <= (uint32_t)kCap ? M_VC : M_VM;
                     }
-                } else if (m0 == M_KH) {
+                } else if (K == 0 && m0 == M_KH) {
                     const uint32_t nlo = lo + (nbin << sh);
                     const uint64_t top = (uint64_t)nlo + ((1ull << sh) - 1ull);
                     hi = top < (uint64_t)hi ? (uint32_t)top : hi;
@@ -590,7 +641,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 bool any = false;
                 uint32_t hit = 0u;
                 if constexpr (WS == 1) {
-                    if (__any_sync(full, cmode)) {
+                    if (K != 1 && __any_sync(full, cmode)) {
                         const uint32_t cmax = __reduce_max_sync(full, cmode ? cnt : 0u);
                         const uint32_t *cl = list + cc * kListStride;
                         for (uint32_t e0 = (uint32_t)g8; e0 < cmax; e0 += 8) {
@@ -608,7 +659,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                             }
                         }
                     }
-                } else if (cmode) {
+                } else if (K != 1 && cmode) {
                     for (uint32_t e0 = (uint32_t)gf; e0 < cnt; e0 += G) {
                         // entry e0 of the concatenated per-warp lists
                         uint32_t m = e0;
@@ -632,9 +683,11 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     }
                 }
                 if constexpr (WS == 1) {
-                    const unsigned mh = __ballot_sync(full, any) & seg;
-                    const uint32_t v = __shfl_sync(full, hit, mh ? __ffs(mh) - 1 : lane);
-                    if (cmode) res = v;
+                    if constexpr (K != 1) {
+                        const unsigned mh = __ballot_sync(full, any) & seg;
+                        const uint32_t v = __shfl_sync(full, hit, mh ? __ffs(mh) - 1 : lane);
+                        if (cmode) res = v;
+                    }
                 } else {
                     if (any) st[3 * TC + cc] = hit;
                     col_sync<WS>(cw);
@@ -642,7 +695,18 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     if (gf == 0) st[4 * TC + cc] = 0u;   // NaN flag, next pass
                     col_sync<WS>(cw);
                 }
-                if (cmode) mode = M_DONE;
+                if (K != 1 && cmode) mode = M_DONE;
+                        };
+            // two lean passes (histogram, list) while every coordinate of the
+            // column is in VH, VC or done; then the general passes, if any
+            pass(std::integral_constant<int, 1>{});
+            pass(std::integral_constant<int, 2>{});
+            if (__builtin_expect((__ballot_sync(full, mode == M_DONE) & 0xfu) != 0xfu, 0)) {
+                for (int k2 = 0; k2 < 20; ++k2) {
+                    // the column's warps hold identical states: the exit is uniform
+                    if ((__ballot_sync(full, mode == M_DONE) & 0xfu) == 0xfu) break;
+                    pass(std::integral_constant<int, 0>{});
+                }
             }
             if (gf == 0 && live) out[c0 + cc] = __uint_as_float(from_key(res));
         }

@@ -322,19 +322,18 @@ def test_generator_torch_cuda_matches_numpy():
 # ------------------------------------------------ exact fallback paths of the median
 
 
-def _median_case(vals):
-    """vals: float32 [n, d] chosen values; run aggregate with one copy per
-    file (r=2, both copies equal) so that every file is kept as is."""
+def _median_case(vals, r=2):
+    """vals: float32 [n, d] chosen values; run aggregate with every copy of a
+    file equal, so that every file is kept as is (rows past n repeat the last)."""
     n, d = vals.shape
-    K = next(k for k in range(2, 200) if math.comb(k, 2) >= n)
-    f = math.comb(K, 2)
-    host = np.zeros((f, 2, d), np.float32)
+    K = next(k for k in range(r, 200) if math.comb(k, r) >= n)
+    f = math.comb(K, r)
+    host = np.zeros((f, r, d), np.float32)
     rows = np.concatenate([vals, np.repeat(vals[-1:], f - n, axis=0)]) if f > n else vals
-    host[:, 0] = rows
-    host[:, 1] = rows
-    oa = oracle.assign(K, 2)
+    host[:] = rows[:, None, :]
+    oa = oracle.assign(K, r)
     want = oracle.run_round(host, oa, d)
-    a = ap.aspis_assign(K, 2)
+    a = ap.aspis_assign(K, r)
     buf = gpu_round(ap, torch, torch.from_numpy(host).to(DEV), d, a)
     assert_round_matches(ap, buf, want)
 
@@ -379,4 +378,80 @@ def test_median_wide_range_and_subnormals():
     n, d = 300, 64
     mag = 10.0 ** rng.uniform(-44, 38, (n, d))
     vals = (rng.choice([-1.0, 1.0], (n, d)) * mag).astype(np.float32)
+    _median_case(vals)
+
+
+# ------------------------------------------- value-space refinement of a crowded bin
+
+
+def _crowd(vals, rng, rows_from, count, spread, ties=0):
+    """Put `count` distinct values within `spread` of each column's median
+    (the first `ties` of them equal to it), away from the sampled rows."""
+    n, d = vals.shape
+    for c in range(d):
+        med = float(np.sort(vals[:, c])[(n - 1) // 2])
+        rows = rng.choice(np.arange(rows_from, n), size=count, replace=False)
+        off = np.linspace(-spread, spread, count)
+        off[:ties] = 0.0
+        vals[rows, c] = (med + off).astype(np.float32)
+
+
+def test_median_refines_crowded_bin():
+    """More than 32 distinct values in the median's bin: one refinement level."""
+    rng = np.random.default_rng(21)
+    vals = rng.standard_normal((455, 96)).astype(np.float32)
+    _crowd(vals, rng, 64, 120, 1e-3)
+    _median_case(vals)
+
+
+def test_median_refines_twice():
+    """A crowd inside the crowd: two refinement levels before the final list."""
+    rng = np.random.default_rng(22)
+    vals = rng.standard_normal((455, 64)).astype(np.float32)
+    _crowd(vals, rng, 64, 200, 1e-2)
+    _crowd(vals, rng, 64, 90, 1e-5)
+    _median_case(vals)
+
+
+def test_median_refine_ties_at_median():
+    """Crowded bin whose members around the target rank are all equal."""
+    rng = np.random.default_rng(23)
+    vals = rng.standard_normal((455, 64)).astype(np.float32)
+    _crowd(vals, rng, 64, 100, 1e-4, ties=70)
+    _median_case(vals)
+
+
+def test_median_crowded_overflow_bin_goes_to_key_space():
+    """The median sits above every sampled value, among values reaching +inf:
+    the members' value range is not finite, so key-space bins take over."""
+    rng = np.random.default_rng(24)
+    n, d = 455, 32
+    vals = np.empty((n, d), np.float32)
+    vals[:16] = rng.uniform(-1.0, 1.0, (16, d))          # the sampled rows
+    big = 10.0 ** rng.uniform(0.5, 38, (n - 16, d))
+    vals[16:] = big.astype(np.float32)
+    vals[rng.choice(np.arange(16, n), 20, replace=False), :] = np.inf
+    _median_case(vals)
+
+
+@pytest.mark.parametrize("r", [3, 5])
+def test_median_refine_many_rows(r):
+    """Thousands of kept files: several warps share a coordinate."""
+    rng = np.random.default_rng(25 + r)
+    n = 2024 if r == 3 else 3003
+    vals = (0.01 * rng.standard_normal((n, 40))).astype(np.float32)
+    _crowd(vals, rng, 256, 300, 1e-5, ties=40)
+    _median_case(vals, r=r)
+
+
+def test_median_values_far_below_a_narrow_sample():
+    """Values some millions of bin widths below the sampled range map to a
+    small negative fma result; they must count in the lowest bin."""
+    rng = np.random.default_rng(27)
+    n, d = 455, 32
+    vals = (1.0 + rng.uniform(0.0, 1.26e-4, (n, d))).astype(np.float32)
+    for c in range(d):
+        rows = rng.choice(np.arange(16, n), 150, replace=False)
+        vals[rows[:100], c] = np.float32(-9.0 - c)
+        vals[rows[100:], c] = np.float32(3.0 + c)
     _median_case(vals)
