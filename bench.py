@@ -230,6 +230,7 @@ def main():
     import numpy as np
     import torch
     import paper_2108_02416_gb300 as ap
+    from paper_2108_02416_gb300.shard import max_over_ranks
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -291,10 +292,7 @@ def main():
     total_ms = t_start.elapsed_time(t_end)
     if flush is not None:         # small inputs: exclude the L2 flush kernels
         total_ms = sum(e[0].elapsed_time(e[3]) for e in evs)
-    if dist:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, dev)     # slowest rank (1 rank: unchanged)
     clocks = clk.summary()
     check_ms = [e[0].elapsed_time(e[1]) for e in evs]
     detsel_ms = [e[1].elapsed_time(e[2]) for e in evs]

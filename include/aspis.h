@@ -130,6 +130,18 @@ aspis_status aspis_check(const float *copies, int64_t d, int64_t ld,
                          const aspis_assignment *a, uint32_t *file_neq,
                          uint32_t *adj, void *stream);
 
+/* Step 2 alone: the graph G from per-file mismatch words (the edge rule of
+ * Algorithm 3, as in aspis_check).  For a PS whose copies are split by
+ * coordinate range over several devices: each device runs aspis_check on
+ * its slice, the file_neq words of all slices are OR-combined (a copy pair
+ * differs iff it differs in some slice), and every device then derives the
+ * same G from the combined words.
+ *   file_neq  device [f] uint32 (slot-pair mismatch words, all bits < r(r-1)/2)
+ *   adj       device [K] uint32, out, as for aspis_check
+ * Reads f*4 bytes.  Overwrites adj entirely. */
+aspis_status aspis_graph(const uint32_t *file_neq, const aspis_assignment *a,
+                         uint32_t *adj, void *stream);
+
 /* Step 3: all maximum cliques of G (Algorithm 3: every maximum clique is
  * listed; exactly one of them means successful detection).  Bron-Kerbosch with pivoting over
  * 32-bit vertex masks in one thread block; each search branch has a node

@@ -79,6 +79,7 @@ def _load():
         "aspis_assignment_to_device": ([A], i32),
         "aspis_assignment_free": ([A], None),
         "aspis_check": ([P, i64, i64, A, P, P, P], i32),
+        "aspis_graph": ([P, A, P, P], i32),
         "aspis_detect": ([P, i32, P, P], i32),
         "aspis_select": ([P, P, A, P, P], i32),
         "aspis_aggregate": ([P, i64, i64, A, P, P, i32, P, P], i32),
@@ -185,6 +186,12 @@ def aspis_check(copies, d: int, a: Assignment, file_neq, adj, stream=None):
     _ok(lib.aspis_check(_dev(copies, torch.float32, "copies"), d, ld, a.ref,
                         _dev(file_neq, torch.int32, "file_neq"), _dev(adj, torch.int32, "adj"),
                         _stream(stream)), "aspis_check")
+
+
+def aspis_graph(file_neq, a: Assignment, adj, stream=None):
+    import torch
+    _ok(lib.aspis_graph(_dev(file_neq, torch.int32, "file_neq"), a.ref,
+                        _dev(adj, torch.int32, "adj"), _stream(stream)), "aspis_graph")
 
 
 def aspis_detect(adj, K: int, det, stream=None):

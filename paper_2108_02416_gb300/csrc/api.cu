@@ -93,6 +93,16 @@ extern "C" aspis_status aspis_check(const float *copies, int64_t d, int64_t ld,
     return cuda_status(launch_graph(file_neq, a->dev_file_workers, a->f, a->r, a->K, adj, st));
 }
 
+extern "C" aspis_status aspis_graph(const uint32_t *file_neq, const aspis_assignment *a,
+                                    uint32_t *adj, void *stream)
+{
+    aspis_status s = check_assignment(a);
+    if (s != ASPIS_OK) return s;
+    if (!file_neq || !adj) return ASPIS_E_INVAL;
+    return cuda_status(launch_graph(file_neq, a->dev_file_workers, a->f, a->r, a->K, adj,
+                                    (cudaStream_t)stream));
+}
+
 extern "C" aspis_status aspis_detect(const uint32_t *adj, int K, aspis_detection *det,
                                      void *stream)
 {

@@ -455,3 +455,54 @@ def test_median_values_far_below_a_narrow_sample():
         vals[rows[:100], c] = np.float32(-9.0 - c)
         vals[rows[100:], c] = np.float32(3.0 + c)
     _median_case(vals)
+
+
+# ------------------------------------------------ coordinate-split round on one GPU
+
+
+def test_graph_entry_point_matches_oracle():
+    w = synth.CONFIGS["k15_r3_d1m_weak_reversed"]
+    oa = oracle.assign(w.K, w.r)
+    a = ap.aspis_assign(w.K, w.r)
+    rng = np.random.default_rng(31)
+    for _ in range(20):
+        words = rng.integers(0, 1 << 3, oa.f).astype(np.uint32) * (rng.random(oa.f) < 0.05)
+        words = words.astype(np.uint32)
+        adj = torch.zeros(w.K, dtype=torch.int32, device=DEV)
+        ap.aspis_graph(torch.from_numpy(words.view(np.int32)).to(DEV), a, adj)
+        torch.cuda.synchronize()
+        want = oracle.graph(oracle.pair_agreement(words, oa), w.K, w.r)
+        assert np.array_equal(as_u32(adj), want)
+
+
+@pytest.mark.parametrize("name", ["k7_r3_d4096_alie", "k15_r3_d11m_strong_alie"])
+def test_coordinate_split_round_equals_whole_round(name):
+    """Two coordinate slices on one device, combined as two ranks would:
+    OR of the mismatch words, then identical graph / cliques / selection and
+    per-slice aggregation.  Must equal the whole round and the oracle."""
+    from paper_2108_02416_gb300 import shard
+    import dataclasses
+    w = dataclasses.replace(synth.CONFIGS[name], d=5000)
+    oa = oracle.assign(w.K, w.r)
+    a = ap.aspis_assign(w.K, w.r)
+    full = torch.from_numpy(synth.build_copies_np(w, oa.file_workers, 0, w.d)).to(DEV)
+    parts = []
+    for p in range(2):
+        c0, c1 = shard.shard_bounds(w.d, 2, p)
+        ops = shard.DeviceOps(a, DEV)
+        parts.append((c0, c1, ops, full[:, :, c0:c1].contiguous()))
+    words = shard.or_combine([ops.compare(x, c1 - c0).clone() for c0, c1, ops, x in parts])
+    outs = []
+    for c0, c1, ops, x in parts:
+        adj = ops.graph(words)
+        det = ops.detect(adj)
+        sel = ops.select(words, det)
+        outs.append(ops.aggregate(x, c1 - c0, sel, det))
+    torch.cuda.synchronize()
+    want = oracle.run_round(full.cpu().numpy(), oa, w.d)
+    assert np.array_equal(as_u32(words), want.file_neq)
+    for c0, c1, ops, x in parts:
+        assert np.array_equal(as_u32(ops.buf.adj), want.adj)
+        assert np.array_equal(ops.buf.sel.cpu().numpy(), want.sel)
+    out = torch.cat(outs).cpu().numpy()
+    assert np.array_equal(out.view(np.uint32), want.out.view(np.uint32))
