@@ -92,7 +92,16 @@ struct Layout {
 };
 
 template <int TC>
-__host__ __device__ constexpr int bin_pitch() { return TC + 4; }   // bytes per row of bins
+__host__ __device__ inline int bin_row(int64_t f)
+{
+    // tag bytes per lane: its rows' tags are contiguous, four per word; an odd
+    // word count puts the 32 lanes of a warp in 32 different banks
+    constexpr int G = 8 * (kWarps / (TC / 4));
+    const int rows = (int)((f + G - 1) / G);
+    int words = (rows + 3) / 4;
+    if ((words & 1) == 0) ++words;
+    return words * 4;
+}
 
 template <int TC, int STAGES>
 __host__ __device__ inline Layout make_layout(int64_t f)
@@ -102,7 +111,7 @@ __host__ __device__ inline Layout make_layout(int64_t f)
     size_t o = 0;
     L.tile_bytes = ((size_t)f * TC * 4 + 127) / 128 * 128;
     L.tiles = o; o += STAGES * L.tile_bytes;
-    L.bins = o; o += ((size_t)(f + 32 * 8 * WS) * bin_pitch<TC>() + 15) / 16 * 16;
+    L.bins = o; o += ((size_t)TC * 8 * WS * bin_row<TC>(f) + 15) / 16 * 16;
     L.rows = o; o += ((size_t)f * 4 + 15) / 16 * 16;
     L.hist = o; o += (size_t)TC * kHistStride * 4;
     L.list = o; o += (size_t)TC * WS * kListStride * 4;
@@ -124,11 +133,10 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     constexpr int RPL = 32 / TC;           // tile rows per 128-byte line
     constexpr int BPL = kNB / G;           // histogram bins summed per lane (16, 8, 4, 2)
     constexpr int RPI = kThreads / CPR;    // tile rows covered by one copy round
-    constexpr int BP = bin_pitch<TC>();
     extern __shared__ __align__(128) unsigned char smem[];
     const Layout L = make_layout<TC, STAGES>(f);
     unsigned char *tiles = smem + L.tiles;
-    uint8_t *bins = smem + L.bins;                                    // [n][BP] bytes
+    uint8_t *bins = smem + L.bins;                                    // [WS][TC][8][JP] tags
     int32_t *rows = reinterpret_cast<int32_t *>(smem + L.rows);
     uint32_t *hist = reinterpret_cast<uint32_t *>(smem + L.hist);     // [TC][kHistStride]
     uint32_t *list = reinterpret_cast<uint32_t *>(smem + L.list);     // [TC][WS][kListStride]
@@ -169,14 +177,12 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     }
     const uint32_t krank = (uint32_t)((n - 1) / 2);
     const int64_t ntiles = (d + TC - 1) / TC;
-    // rows past n read as bin 0xFF, which no value has (bins are < kNB)
-    for (int e = tid; e < 32 * G * BP; e += kThreads) bins[n * BP + e] = 0xFFu;
 
     // lane's first element (in words) and the stride between its rows
     const int fl = (gf / RPL) & (CPR - 1);
     const int off0 = gf * TC + ((cw ^ fl) << 2) + cq;
     constexpr int kStride = G * TC;
-    constexpr int kBStride = G * BP;
+    const int JP = bin_row<TC>(f);
     const int nmine = n > gf ? (n - gf + G - 1) / G : 0;
 
     // copy role (vector path): this thread always moves chunk ch_me of rows
@@ -222,12 +228,22 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     };
 
     const int64_t t0 = blockIdx.x;
+    // One stage: the next tile is fetched into the same buffer as soon as this
+    // one is no longer read (after the list pass, when no coordinate needs
+    // the general passes), else at the end of the tile.  More stages: tile
+    // t + (STAGES-1) grids is fetched when tile t starts.
+    if constexpr (STAGES == 1) {
+        issue(t0, 0);
+    } else {
 #pragma unroll
-    for (int s = 0; s < STAGES - 1; ++s) issue(t0 + (int64_t)s * gridDim.x, s);
+        for (int s = 0; s < STAGES - 1; ++s) issue(t0 + (int64_t)s * gridDim.x, s);
+    }
 
     int stage = 0;
     for (int64_t t = t0; t < ntiles; t += gridDim.x) {
-        issue(t + (int64_t)(STAGES - 1) * gridDim.x, (stage + STAGES - 1) % STAGES);
+        if constexpr (STAGES > 1)
+            issue(t + (int64_t)(STAGES - 1) * gridDim.x, (stage + STAGES - 1) % STAGES);
+        bool fetched = false;             // the next tile is on its way (one stage)
         cp_async_wait<STAGES - 1>();
         __syncthreads();
         uint32_t *tile = reinterpret_cast<uint32_t *>(tiles + stage * L.tile_bytes);
@@ -312,7 +328,8 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             int mode = !live ? M_DONE : (vspace ? M_VH : M_KA);
             uint32_t lo = 0u, hi = 0u, krem = krank, cnt = (uint32_t)n, res = 0u, vb = 0u;
             int vr_levels = 0;
-            uint8_t *bmine = bins + gf * BP + cc;       // this lane's first bin byte
+            // this lane's tags, one byte per row, contiguous
+            uint8_t *bmine = bins + ((ws * TC + cc) * 8 + g8) * JP;
 
             auto pass = [&](auto kind) {
 
@@ -333,9 +350,9 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 uint32_t amin = 0xffffffffu, amax = 0u;
                 bool nanf = false;
                 if (K != 2 && m0 == M_VH) {
-                    uint8_t *pb = bmine;
+                    uint32_t *pb = reinterpret_cast<uint32_t *>(bmine);
                     int j = 0;
-                    for (; j + 4 <= nmine; j += 4, p += 4 * kStride, pb += 4 * kBStride) {
+                    for (; j + 4 <= nmine; j += 4, p += 4 * kStride, ++pb) {
                         const float y0 = fmaf(__uint_as_float(p[0]), vs, vc);
                         const float y1 = fmaf(__uint_as_float(p[kStride]), vs, vc);
                         const float y2 = fmaf(__uint_as_float(p[2 * kStride]), vs, vc);
@@ -346,17 +363,19 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                         atomicAdd(h + b1, 1u);
                         atomicAdd(h + b2, 1u);
                         atomicAdd(h + b3, 1u);
-                        pb[0] = (uint8_t)b0;
-                        pb[kBStride] = (uint8_t)b1;
-                        pb[2 * kBStride] = (uint8_t)b2;
-                        pb[3 * kBStride] = (uint8_t)b3;
+                        *pb = b0 | (b1 << 8) | (b2 << 16) | (b3 << 24);
                     }
-                    for (; j < nmine; ++j, p += kStride, pb += kBStride) {
-                        const float y = fmaf(__uint_as_float(*p), vs, vc);
-                        nanf |= y != y;
-                        const uint32_t b = vbin(y);
-                        atomicAdd(h + b, 1u);
-                        *pb = (uint8_t)b;
+                    if (j < nmine) {
+                        // last, partial word: missing rows get tag 0xFF, which no bin has
+                        uint32_t word = 0xFFFFFFFFu;
+                        for (int q = 0; j < nmine; ++j, ++q, p += kStride) {
+                            const float y = fmaf(__uint_as_float(*p), vs, vc);
+                            nanf |= y != y;
+                            const uint32_t b = vbin(y);
+                            atomicAdd(h + b, 1u);
+                            word = (word & ~(0xFFu << (8 * q))) | (b << (8 * q));
+                        }
+                        *pb = word;
                     }
                 }
                 if constexpr (K == 0) {
@@ -373,38 +392,48 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     }
                 }
                 }
-                // VC: byte compare into per-lane masks of 32 rows, then the
-                // members are stored at a prefix over the coordinate's lanes
+                // VC: one 32-bit load tests four of the lane's rows against the
+                // bin; members are counted, stored at a prefix over the
+                // coordinate's lanes, and only the words holding one are revisited
                 if constexpr (K != 1) {
                 if (__any_sync(full, m0 == M_VC)) {
                     uint32_t *lst = list + (cc * WS + ws) * kListStride;
-                    const int iters = (int)__reduce_max_sync(full, m0 == M_VC ? (unsigned)nmine : 0u);
-                    uint32_t nlist = 0u;
-                    for (int jb = 0; jb < iters; jb += 32) {
-                        const uint8_t *pb = bmine + jb * kBStride;
-                        uint32_t mask = 0u;
-#pragma unroll
-                        for (int jj = 0; jj < 32; ++jj)
-                            mask |= (pb[jj * kBStride] == vb ? 1u : 0u) << jj;
-                        if (m0 != M_VC) mask = 0u;
-                        const uint32_t cntm = __popc(mask);
-                        uint32_t incl = cntm;
-#pragma unroll
-                        for (int o = 1; o < 8; o <<= 1) {
-                            const uint32_t tv = __shfl_up_sync(full, incl, 4 * o);
-                            if (g8 >= o) incl += tv;
-                        }
-                        const uint32_t tot = __shfl_sync(full, incl, 28 + cq);
-                        uint32_t pos = nlist + incl - cntm;
-                        while (mask) {
-                            const int jj = __ffs(mask) - 1;
-                            mask &= mask - 1;
-                            lst[pos++] = to_key(tile[off0 + (jb + jj) * kStride]);
-                        }
-                        nlist += tot;
+                    const uint32_t *pw = reinterpret_cast<const uint32_t *>(bmine);
+                    const uint32_t vbx = vb * 0x01010101u;
+                    const int nw = m0 == M_VC ? (nmine + 3) >> 2 : 0;
+                    uint32_t nm = 0u, wm = 0u;
+#pragma unroll 4
+                    for (int q = 0; q < nw; ++q) {
+                        const uint32_t z = tag_match(pw[q], vbx);
+                        nm += __popc(z);
+                        wm |= (q < 32 && z != 0u) ? 1u << q : 0u;
                     }
-                    if (m0 == M_VC && g8 == 0) lcnt[cc * WS + ws] = nlist;
+                    uint32_t incl = nm;
+#pragma unroll
+                    for (int o = 1; o < 8; o <<= 1) {
+                        const uint32_t tv = __shfl_up_sync(full, incl, 4 * o);
+                        if (g8 >= o) incl += tv;
+                    }
+                    const uint32_t tot = __shfl_sync(full, incl, 28 + cq);
+                    uint32_t pos = incl - nm;
+                    for (; wm; wm &= wm - 1) {
+                        const int q = __ffs(wm) - 1;
+                        for (uint32_t z = tag_match(pw[q], vbx); z; z &= z - 1)
+                            lst[pos++] = to_key(tile[off0 + (q * 4 + ((__ffs(z) - 1) >> 3)) * kStride]);
+                    }
+                    for (int q = 32; q < nw; ++q)            // rows past 128 of a lane
+                        for (uint32_t z = tag_match(pw[q], vbx); z; z &= z - 1)
+                            lst[pos++] = to_key(tile[off0 + (q * 4 + ((__ffs(z) - 1) >> 3)) * kStride]);
+                    if (m0 == M_VC && g8 == 0) lcnt[cc * WS + ws] = tot;
                 }
+                }
+                if constexpr (K == 2 && STAGES == 1) {
+                    // every warp is past the tile unless a coordinate still
+                    // needs the general passes (which read it)
+                    if (!__syncthreads_or(m0 != M_VC && m0 != M_DONE)) {
+                        issue(t + gridDim.x, 0);
+                        fetched = true;
+                    }
                 }
                 if constexpr (K == 0) {
                 // VM: key range of the members of bin vb (too many to list)
@@ -412,7 +441,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     uint32_t kmin = 0xffffffffu, kmax = 0u;
                     if (m0 == M_VM)
                         for (int j = 0; j < nmine; ++j)
-                            if (bmine[j * kBStride] == vb) {
+                            if (bmine[j] == vb) {
                                 const uint32_t k = to_key(tile[off0 + j * kStride]);
                                 kmin = min(kmin, k);
                                 kmax = max(kmax, k);
@@ -456,7 +485,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 // every other tag becomes 0xFF, which no bin has
                 if (m0 == M_VR) {
                     uint8_t *pbr = bmine;
-                    for (int j = 0; j < nmine; ++j, pbr += kBStride) {
+                    for (int j = 0; j < nmine; ++j, ++pbr) {
                         uint32_t b = 0xFFu;
                         if (*pbr == vb) {
                             b = vbin(fmaf(__uint_as_float(tile[off0 + j * kStride]), rs, rc));
@@ -710,7 +739,10 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             }
             if (gf == 0 && live) out[c0 + cc] = __uint_as_float(from_key(res));
         }
-        __syncthreads();
+        if (!fetched) {
+            __syncthreads();
+            if constexpr (STAGES == 1) issue(t + gridDim.x, 0);
+        }
         stage = (stage + 1) % STAGES;
     }
     cp_async_wait<0>();

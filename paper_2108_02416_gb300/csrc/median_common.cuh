@@ -1,5 +1,5 @@
 // Pieces of the lower-median search (aggregate.cu): the totalOrder key map,
-// the value-space bin map and the search modes.
+// the value-space bin map, tag matching and the search modes.
 #pragma once
 
 #include <stdint.h>
@@ -36,6 +36,16 @@ __device__ __forceinline__ uint32_t vbin(float y)
 }
 
 enum { M_DONE = 0, M_VH, M_VC, M_VM, M_VR, M_KA, M_KH, M_KC };
+
+// Four tag bytes against the replicated bin vbx: 0x80 in each byte whose tag
+// equals the bin.  Tags are < 0x80 and padding is 0xFF, so after the XOR a
+// byte is zero exactly at a match; OR-ing 0x80 first keeps the per-byte
+// subtraction from borrowing across bytes.
+__device__ __forceinline__ uint32_t tag_match(uint32_t word, uint32_t vbx)
+{
+    const uint32_t x = word ^ vbx;
+    return ~((x | 0x80808080u) - 0x01010101u) & ~x & 0x80808080u;
+}
 
 // Two-sum: s + e == a + b exactly (Knuth); no products, so nothing to fuse.
 __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e)
