@@ -188,6 +188,38 @@ aspis_status aspis_round(const float *copies, int64_t d, int64_t ld,
                          uint32_t *adj, aspis_detection *det, int8_t *sel,
                          int mode, float *out, void *stream);
 
+/* Largest f accepted by aspis_round_static, and the size in bytes of the
+ * fixed device array that holds its per-round intermediates. */
+#define ASPIS_STATIC_MAX_FILES 6144
+#define ASPIS_STATIC_SCRATCH_BYTES 81920
+
+/* aspis_round for callers that cannot allocate device memory.  The paper has
+ * no counterpart: this is a deployment variant of the same round.  Callers
+ * such as runtimes that hand the library buffers from their own memory pool,
+ * or processes whose allocator is locked or budgeted, may own the copies,
+ * the output and the detection record but cannot let a library call
+ * cudaMalloc (aspis_assignment_to_device does; aspis_round needs caller
+ * buffers for file_neq, adj and sel).  This call allocates nothing: the
+ * mismatch words, the graph, the selection and a device copy of the
+ * assignment table live in one file-scope device array of
+ * ASPIS_STATIC_SCRATCH_BYTES bytes, which every GPU that loads the library
+ * holds until the process exits.
+ *   copies  device [f][r][ld] fp32, as for aspis_round
+ *   a       host tables from aspis_assign; the device mirror is not needed
+ *           (file_workers is copied into the array on the stream every call)
+ *   det     device aspis_detection, out, as for aspis_round
+ *   out     device [d] fp32, out; mode as for aspis_aggregate
+ * Results equal aspis_round's.  f > ASPIS_STATIC_MAX_FILES returns
+ * ASPIS_E_RANGE before anything is enqueued.  The first call on a device
+ * looks up the array's device address (cudaGetSymbolAddress, with that
+ * device current); make that first call before any stream capture.  All
+ * calls share the array and its contents persist between calls (the parts
+ * that must start at zero are cleared by each call): calls that may overlap
+ * on the GPU, e.g. on unordered streams, race and must not be issued. */
+aspis_status aspis_round_static(const float *copies, int64_t d, int64_t ld,
+                                const aspis_assignment *a, aspis_detection *det,
+                                int mode, float *out, void *stream);
+
 /* The whole round from host memory: copies the f*r*ld floats at
  * host_copies (pinned memory gives full bandwidth) into the device buffer
  * dev_copies, runs aspis_round, and copies the d aggregated floats into

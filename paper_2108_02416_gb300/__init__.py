@@ -15,6 +15,7 @@ The call names mirror the C entry points:
   aspis_aggregate(copies, d, a, sel, det, out, mode)   coordinate-wise median / mean
   aspis_round(...)                          the four device steps on one stream
   aspis_round_host(...)                     the same from pinned host memory
+  aspis_round_static(copies, d, a, det, out, mode)   the round with no device allocation
 """
 from __future__ import annotations
 
@@ -26,6 +27,7 @@ LIB_PATH = os.path.join(PKG, "libaspis.so")
 
 OK, E_INVAL, E_RANGE, E_ALIGN, E_CUDA, E_LIMIT, E_EMPTY, E_NOT_IMPLEMENTED = range(8)
 MAX_K, MAX_R, MAX_AGG_FILES = 31, 8, 6144
+STATIC_MAX_FILES = 6144
 MEDIAN, MEAN = 0, 1
 
 
@@ -85,6 +87,7 @@ def _load():
         "aspis_aggregate": ([P, i64, i64, A, P, P, i32, P, P], i32),
         "aspis_round": ([P, i64, i64, A, P, P, P, P, i32, P, P], i32),
         "aspis_round_host": ([P, P, i64, i64, A, P, P, P, P, i32, P, P, P, P], i32),
+        "aspis_round_static": ([P, i64, i64, A, P, i32, P, P], i32),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -242,6 +245,18 @@ def aspis_round_host(host_copies, dev_copies, d: int, a: Assignment, file_neq, a
                              ctypes.c_void_p(host_out.data_ptr()),
                              ctypes.c_void_p(host_det.data_ptr()), _stream(stream)),
         "aspis_round_host")
+
+
+def aspis_round_static(copies, d: int, a: Assignment, det, out, mode: int = MEDIAN, stream=None):
+    """The round for callers that cannot allocate device memory: the
+    intermediates live in the library's fixed device array (see aspis.h);
+    ``a`` needs no device mirror.  Calls that may overlap on the GPU race."""
+    import torch
+    ld = _ld(copies, a)
+    _ok(lib.aspis_round_static(_dev(copies, torch.float32, "copies"), d, ld, a.ref,
+                               _dev(det, torch.uint8, "det"), mode,
+                               _dev(out, torch.float32, "out"), _stream(stream)),
+        "aspis_round_static")
 
 
 class RoundBuffers:
