@@ -1,44 +1,46 @@
 // Step 5 of the PS round: coordinate-wise aggregation of the chosen copies
 // (Algorithm 1: median of the majority gradients; mean in Case 1).
 //
-// Layout.  A tile is TC consecutive coordinates (TC = 32, 16, 8 or 4) of all
-// n kept rows, staged row-major in shared memory ([row][TC] floats) by
-// 16-byte cp.async copies, TC/4 consecutive threads per row, so every
-// request carries the row's whole TC*4-byte segment.  Lane l of a warp works
-// on coordinate c = l % TC of the tile; the SUB = 32/TC lanes of a warp that
-// share a coordinate and the 8 warps split its rows: thread (w, s) owns slot
-// w*SUB + s and rows slot, slot + NS, slot + 2*NS, ... (NS = 8*SUB slots).
-// With this assignment every shared access of the per-value loops is free of
-// bank conflicts by construction: the 32 lanes of a load read 32 consecutive
-// words of the tile; each lane counts into its own histogram column (bank =
-// lane); tag words are laid out [word][slot][TC].  Two CTAs share an SM, or
-// one CTA keeps STAGES tiles in flight.
+// Data path.  A tile is TC = 32*V consecutive coordinates (V = 4, 2 or 1) of
+// all n kept rows.  Lane l of every warp holds coordinates [l*V, l*V + V) of
+// the tile and the 8 warps split the rows: warp w reads rows w, w + 8, ...
+// straight from global memory with one V-wide load per row, so a warp-wide
+// load is one contiguous 128*V-byte segment of a row.  (Gathering 128-byte
+// segments of 455 rows that lie 45 MB apart runs at about 4.9 TB/s on GB300,
+// 512-byte segments at 7.0; staging whole tiles in shared memory would limit
+// the segments to 128 bytes.)  Each value is used once, from registers: rows
+// come in batches of kU per thread, every register refilled with the next
+// batch's row as soon as it is read, and the last batch of a tile refills
+// with the first rows of the CTA's next tile, whose loads then overlap this
+// tile's remaining phases.  Shared memory holds one tag byte per value, the
+// histograms and small per-coordinate state; two CTAs share an SM.
 //
-// Lower median, exact (IEEE totalOrder through a monotone uint32 key; the
-// key map is a bijection, so the output has the chosen element's bits).  Per
+// Lower median, exact (IEEE totalOrder through a monotone uint32 key; the key
+// map is a bijection, so the output has the chosen element's bits).  Per
 // tile:
-//   S   sample: the key range [min, max] of the first two values of every
-//       slot (16 values per coordinate for TC = 32).
-//   VH  value-space histogram of all values: 128 bins, bins 1..126 evenly
-//       over the sample range, 0 / 127 catching everything below / above.
-//       The bin map x -> bits(fma(x, s, c)) - bits(2^23), clamped, is
-//       monotone in totalOrder, so bins are contiguous value ranges.  Every
-//       value's bin is kept as a tag byte.  NaNs are detected on the way.
-//   B   bin search: per-slot partial sums over the bins, then the slot whose
-//       bins hold the target rank finds the bin, the rank inside it and its
-//       count (bins of one slot stay in its registers).
-//   VC  the bin's members (found by comparing four tag bytes per word) are
-//       written to a per-coordinate list of at most 32 keys; each candidate
-//       is ranked against the list directly.
-// Exact fallback, for the coordinates that need it (NaN seen, degenerate or
-// non-finite sample range, more than 32 members in the target bin):
-//   VM  the exact key range [lo, hi] of the crowded bin's members
-//   KA  the key range [lo, hi] of all values
+//   S   sample: key range of the first two rows of every warp (16 values per
+//       coordinate).
+//   VH  value-space histogram of every value: bins 1..125 evenly over the
+//       sample range, 0 and 126 catch everything below / above (vbin_bits);
+//       each value's bin is kept as a tag byte; NaNs are detected.  Counters
+//       are the 16-bit halves of words in per-lane columns, so the 32 shared
+//       atomics of a warp instruction hit 32 different banks.
+//   B   bin search: per-warp partial sums over 16 bins, then one thread per
+//       coordinate finds the bin that holds the target rank, the rank inside
+//       it and its count.
+//   VC  four tag bytes are compared per word; the bin's members (about n/100)
+//       are re-read from global memory (L2) into a list of at most kCap keys
+//       per coordinate, which 8 threads per coordinate rank directly.
+// Exact fallback for the coordinates that need it (NaN seen, degenerate or
+// non-finite sample range, more than kCap members in the bin), values
+// re-read from global memory:
+//   VM  exact key range [lo, hi] of the crowded bin's members
+//   KA  key range [lo, hi] of all values
 //   KH  128 equal-width key-space bins over [lo, hi]; the bin holding the
 //       rank becomes [lo, hi] (each pass shrinks the range by 2^7)
-//   KC  the at most 32 keys left in [lo, hi] are listed and ranked.
+//   KC  the at most kCap keys left in [lo, hi] are listed and ranked.
 // The fallback loop is bounded (kMaxPasses); every wait is a block barrier.
-#include <climits>
+#include <type_traits>
 
 #include "aspis_internal.cuh"
 #include "median_common.cuh"
@@ -46,44 +48,77 @@
 namespace aspis {
 namespace {
 
-constexpr int kThreads = 256;     // 8 warps
-constexpr int kWarps = kThreads / 32;
-constexpr int kMaxPasses = 12;    // fallback passes: KA/VM, at most 5 KH, KC
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;     // row slots of a CTA
+constexpr int kU = 8;                     // rows per load batch and thread
+constexpr int kMaxPasses = 12;            // fallback: VM/KA, at most 5 KH, KC
 
-// per-coordinate state words (arrays of TC words in shared memory)
-enum { S_SMIN, S_SMAX, S_NAN, S_LCNT, S_BIN, S_REM, S_CNT, S_KMIN, S_KMAX, kStateWords };
+// per-coordinate state, arrays of TC words
+enum { S_MIN, S_MAX, S_NAN, S_LCNT, S_MODE, S_BIN, S_REM, S_CNT, S_LO, S_HI, S_PCNT, S_PREM,
+       kStateWords };
+// S_PCNT / S_PREM: count and rank of the listed bin of the pending tile
+// (S_PCNT = 0: nothing to rank for that coordinate)
 
-template <int TC>
-struct Geo {
-    static constexpr int SUB = 32 / TC;          // lanes of a warp on one coordinate
-    static constexpr int NS = kWarps * SUB;      // row slots of a CTA
-    static constexpr int CPR = TC / 4;           // 16-byte chunks per tile row
-    static constexpr int RPI = kThreads / CPR;   // tile rows per copy round
-    static constexpr int BPT = kNB / NS;         // bins per slot in the bin search
-    static constexpr int VS = NS * TC;           // words between a lane's consecutive rows
-};
+template <int V> struct Vec;
+template <> struct Vec<4> { using T = uint4; };
+template <> struct Vec<2> { using T = uint2; };
+template <> struct Vec<1> { using T = uint32_t; };
 
-__device__ __forceinline__ void cp_async16(uint32_t saddr, const void *g)
+template <int V>
+__device__ __forceinline__ uint32_t elem(const typename Vec<V>::T &x, int k)
 {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(saddr), "l"(g));
+    if constexpr (V == 4) return k == 0 ? x.x : k == 1 ? x.y : k == 2 ? x.z : x.w;
+    else if constexpr (V == 2) return k == 0 ? x.x : x.y;
+    else return x;
+}
+
+template <int V>
+__device__ __forceinline__ typename Vec<V>::T load_row(const float *p)
+{
+    if constexpr (V == 4) return __ldcg(reinterpret_cast<const uint4 *>(p));
+    else if constexpr (V == 2) return __ldcg(reinterpret_cast<const uint2 *>(p));
+    else return __ldcg(reinterpret_cast<const unsigned int *>(p));
+}
+
+template <uint32_t INC>
+__device__ __forceinline__ void red_shared(uint32_t saddr)
+{
+    asm volatile("red.shared.add.u32 [%0], %1;\n" ::"r"(saddr), "n"(INC) : "memory");
 }
 
 __device__ __forceinline__ void cp_async4(uint32_t saddr, const void *g)
 {
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(saddr), "l"(g));
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(saddr), "l"(g) : "memory");
 }
 
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
 
-// max that propagates NaN: a NaN anywhere in the chain survives
-__device__ __forceinline__ float max_nan(float a, float b)
+// ascending bitonic sorting network over 16 registers
+__device__ __forceinline__ void sort16(uint32_t (&y)[16])
 {
-    float r;
-    asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
-    return r;
+#pragma unroll
+    for (int k = 2; k <= 16; k <<= 1)
+#pragma unroll
+        for (int j = k >> 1; j > 0; j >>= 1)
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                const int l = i ^ j;
+                if (l > i) {
+                    const uint32_t a = y[i], b = y[l];
+                    const bool up = (i & k) == 0;
+                    y[i] = up ? min(a, b) : max(a, b);
+                    y[l] = up ? max(a, b) : min(a, b);
+                }
+            }
+}
+
+// flag |= 1 if any of a, b, c, e is NaN (one compare per pair)
+__device__ __forceinline__ void nan_check(uint32_t &flag, float a, float b, float c, float e)
+{
+    asm("{\n .reg .pred p;\n setp.nan.f32 p, %1, %2;\n setp.nan.or.f32 p, %3, %4, p;\n"
+        " @p mov.b32 %0, 1;\n}\n" : "+r"(flag) : "f"(a), "f"(b), "f"(c), "f"(e));
 }
 
 // the low bytes of four words, packed into one word
@@ -92,55 +127,57 @@ __device__ __forceinline__ uint32_t pack4(uint32_t b0, uint32_t b1, uint32_t b2,
     return __byte_perm(__byte_perm(b0, b1, 0x0040), __byte_perm(b2, b3, 0x0040), 0x5410);
 }
 
-struct Layout {
-    size_t tiles, tile_bytes, tags, hist, part, list, state, rows, total;
-    int jw;                       // tag words per slot
+template <int V>
+struct Geo {
+    static constexpr int TC = 32 * V;                 // coordinates per tile
+    static constexpr int NP = V >= 2 ? V / 2 : 1;     // histogram words per (bin, lane)
+    static constexpr int SHB = NP == 2 ? 8 : 7;       // log2 of the bytes per histogram row
+    static constexpr int RPW = 4 / V;                 // rows per tag word
 };
 
-template <int TC, int STAGES>
+struct Layout {
+    size_t tags, hist, list, state, rows, total;
+};
+
+template <int V>
 __host__ __device__ inline Layout make_layout(int64_t f)
 {
-    using G = Geo<TC>;
+    using G = Geo<V>;
     Layout L{};
-    const int64_t per_slot = (f + G::NS - 1) / G::NS;
-    L.jw = (int)((per_slot + 3) / 4);
+    const int64_t per_slot = (f + kWarps - 1) / kWarps;
+    const int64_t jw = (per_slot + G::RPW - 1) / G::RPW;     // tag words per thread
     size_t o = 0;
-    L.tile_bytes = ((size_t)f * TC * 4 + 127) / 128 * 128;
-    L.tiles = o; o += STAGES * L.tile_bytes;
-    L.tags = o; o += (size_t)L.jw * G::VS * 4;
-    L.hist = o; o += (size_t)kNB * 32 * 4;
-    L.part = o; o += (size_t)2 * G::NS * TC * 4;
-    L.list = o; o += (size_t)kCap * TC * 4;
-    L.state = o; o += (size_t)kStateWords * TC * 4;
-    L.rows = o; o += ((size_t)f * 4 + 15) / 16 * 16;
+    L.tags = o; o += (size_t)jw * kWarps * 32 * 4;
+    L.hist = o; o += (size_t)kNB * G::NP * 32 * 4;
+    L.list = o; o += (size_t)kCap * G::TC * 4;       // also the bin-search and mean partials
+    L.state = o; o += (size_t)kStateWords * G::TC * 4;
+    L.rows = o; o += ((size_t)f * 2 + 15) / 16 * 16;
     L.total = o;
     return L;
 }
 
-template <int TC, int STAGES, int MINB, bool VEC, int MODE>
+template <int V, int MINB, bool W32, int MODE>
 __global__ void __launch_bounds__(kThreads, MINB)
 aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, int64_t ld,
                  const int8_t *__restrict__ sel, aspis_detection *det, float *__restrict__ out)
 {
-    using G = Geo<TC>;
-    constexpr int SUB = G::SUB, NS = G::NS, CPR = G::CPR, RPI = G::RPI, BPT = G::BPT;
-    constexpr int VS = G::VS;
-    extern __shared__ __align__(128) unsigned char smem[];
-    const Layout L = make_layout<TC, STAGES>(f);
-    unsigned char *tiles = smem + L.tiles;
-    uint32_t *tags = reinterpret_cast<uint32_t *>(smem + L.tags);    // [jw][NS][TC]
-    uint32_t *hist = reinterpret_cast<uint32_t *>(smem + L.hist);    // [kNB][32]
-    uint32_t *part = reinterpret_cast<uint32_t *>(smem + L.part);    // [2][NS][TC]
-    uint32_t *list = reinterpret_cast<uint32_t *>(smem + L.list);    // [kCap][TC]
-    uint32_t *st = reinterpret_cast<uint32_t *>(smem + L.state);     // [kStateWords][TC]
-    int32_t *rows = reinterpret_cast<int32_t *>(smem + L.rows);
+    using G = Geo<V>;
+    using T = typename Vec<V>::T;
+    constexpr int TC = G::TC, NP = G::NP, SHB = G::SHB, RPW = G::RPW;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const Layout L = make_layout<V>(f);
+    uint32_t *tags = reinterpret_cast<uint32_t *>(smem + L.tags);     // [word][kWarps][32]
+    uint32_t *hist = reinterpret_cast<uint32_t *>(smem + L.hist);     // [kNB][NP][32]
+    uint32_t *list = reinterpret_cast<uint32_t *>(smem + L.list);     // [kCap][TC]
+    uint32_t *st = reinterpret_cast<uint32_t *>(smem + L.state);      // [kStateWords][TC]
+    uint16_t *rows = reinterpret_cast<uint16_t *>(smem + L.rows);
     __shared__ int warp_tot[kWarps];
 
     const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
-    const int c = lane % TC, s = lane / TC;
-    const int slot = w * SUB + s;
     const unsigned full = 0xffffffffu;
-    auto S = [&](int k) -> uint32_t & { return st[k * TC + c]; };
+    const uint32_t hist_s = (uint32_t)__cvta_generic_to_shared(hist);
+    const uint32_t list_s = (uint32_t)__cvta_generic_to_shared(list);
+    auto S = [&](int k, int c) -> uint32_t & { return st[k * TC + c]; };
 
     // ---- kept files: rows[k] = i*r + sel[i] for the k-th file with sel >= 0
     int n = 0;
@@ -155,7 +192,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             off += q < w ? warp_tot[q] : 0;
             tot += warp_tot[q];
         }
-        if (sv >= 0) rows[off + __popc(m & ((1u << lane) - 1u))] = (int32_t)(i * r + sv);
+        if (sv >= 0) rows[off + __popc(m & ((1u << lane) - 1u))] = (uint16_t)(i * r + sv);
         n += tot;
         __syncthreads();
     }
@@ -164,380 +201,471 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
         return;
     }
     const uint32_t krank = (uint32_t)((n - 1) / 2);
+    const int nmine = n > w ? (n - w + kWarps - 1) / kWarps : 0;     // rows of this warp
+    const int nwords = (nmine + RPW - 1) / RPW;
     const int64_t ntiles = (d + TC - 1) / TC;
-    const int nmine = n > slot ? (n - slot + NS - 1) / NS : 0;   // rows of this slot
+    const uint64_t ldb = (uint64_t)ld * 4u;                          // row pitch in bytes
 
-    if constexpr (MODE == 0) {
-        for (int i = tid * 4; i < kNB * 32; i += kThreads * 4)
-            *reinterpret_cast<uint4 *>(hist + i) = make_uint4(0u, 0u, 0u, 0u);
-        if (tid < TC) {
-            st[S_SMIN * TC + tid] = 0xffffffffu;
-            st[S_SMAX * TC + tid] = 0u;
-            st[S_NAN * TC + tid] = 0u;
-            st[S_LCNT * TC + tid] = 0u;
-            st[S_KMIN * TC + tid] = 0xffffffffu;
-            st[S_KMAX * TC + tid] = 0u;
-        }
+    for (int i = tid; i < TC; i += kThreads) {
+        S(S_MIN, i) = 0xffffffffu;
+        S(S_MAX, i) = 0u;
+        S(S_NAN, i) = 0u;
+        S(S_LCNT, i) = 0u;
+        S(S_PCNT, i) = 0u;
     }
+    for (int i = tid * 4; i < kNB * NP * 32; i += kThreads * 4)
+        *reinterpret_cast<uint4 *>(hist + i) = make_uint4(0u, 0u, 0u, 0u);
 
-    // copy role (vector path): this thread moves chunk ch_me of rows i0_me + RPI*k
-    const int ch_me = tid % CPR, i0_me = tid / CPR;
+    // address of row j of this warp at the lane's chunk of a tile
+    auto row_ptr = [&](const char *lb, int j) -> const float * {
+        const uint32_t row = rows[w + j * kWarps];
+        if constexpr (W32) return reinterpret_cast<const float *>(lb + (uint64_t)row * (uint32_t)ldb);
+        else return reinterpret_cast<const float *>(lb + (uint64_t)row * ldb);
+    };
+    auto lane_base = [&](int64_t t) -> const char * {
+        return reinterpret_cast<const char *>(copies + t * TC + lane * V);
+    };
 
-    auto issue = [&](int64_t t, int stage) {
-        if (t < ntiles) {
-            const int64_t c0 = t * TC;
-            const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(tiles + stage * L.tile_bytes);
-            if constexpr (VEC) {
-                const int64_t cg = c0 + ch_me * 4;
-                if (cg < d) {
-                    const float *src = copies + cg;
-                    uint32_t dst = sbase + (uint32_t)(i0_me * TC + ch_me * 4) * 4u;
-                    int i = i0_me;
-                    for (; i + 3 * RPI < n; i += 4 * RPI, dst += 4 * RPI * TC * 4) {
-                        const int32_t r0 = rows[i], r1 = rows[i + RPI];
-                        const int32_t r2 = rows[i + 2 * RPI], r3 = rows[i + 3 * RPI];
-                        cp_async16(dst, src + (int64_t)r0 * ld);
-                        cp_async16(dst + RPI * TC * 4, src + (int64_t)r1 * ld);
-                        cp_async16(dst + 2 * RPI * TC * 4, src + (int64_t)r2 * ld);
-                        cp_async16(dst + 3 * RPI * TC * 4, src + (int64_t)r3 * ld);
-                    }
-                    for (; i < n; i += RPI, dst += RPI * TC * 4)
-                        cp_async16(dst, src + (int64_t)rows[i] * ld);
-                }
+    T xa[kU];                            // the batch being processed (then the next one)
+    {
+        const int64_t t = blockIdx.x;
+        const bool lv = t < ntiles && t * TC + lane * V < d;
+#pragma unroll
+        for (int u = 0; u < kU; ++u)
+            xa[u] = (lv && u < nmine) ? load_row<V>(row_ptr(lane_base(t), u)) : T{};
+    }
+    __syncthreads();
+
+    // The previous tile ("pending"): its median bins are known, its members
+    // are listed during the next sweep and ranked after it.
+    bool have_p = false;
+    const char *lb_p = nullptr;
+    int64_t c0_p = 0;
+    uint32_t vbx_p = 0xFFFFFFFFu, vcm_p = 0u;
+
+    // members of the pending tile among the four tag bytes of word q: their
+    // values are copied (4-byte cp.async) into the coordinate's list column
+    auto capture = [&](uint32_t z, int q) {
+        for (; z; z &= z - 1u) {
+            const int pos = (__ffs(z) - 1) >> 3;
+            const int j = q * RPW + pos / V, k = pos % V;
+            if (j < nmine && ((vcm_p >> k) & 1u)) {
+                const int c = lane * V + k;
+                const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
+                if (at < (uint32_t)kCap)
+                    cp_async4(list_s + (at * TC + c) * 4u, row_ptr(lb_p, j) + k);
+            }
+        }
+    };
+
+    // rank the pending tile's listed bins: one thread per coordinate
+    auto rank_pending = [&]() {
+        for (int c = tid; c < TC; c += kThreads) {
+            const uint32_t cnt = S(S_PCNT, c);
+            if (cnt == 0u) continue;
+            const uint32_t rk = S(S_PREM, c);
+            uint32_t res = 0u;
+            if (cnt <= 16u) {
+                uint32_t y[16];
+#pragma unroll
+                for (int e = 0; e < 16; ++e) y[e] = (uint32_t)e < cnt ? to_key(list[e * TC + c]) : 0xffffffffu;
+                sort16(y);
+                res = y[0];
+#pragma unroll
+                for (int e = 1; e < 16; ++e) res = (uint32_t)e == rk ? y[e] : res;
             } else {
-                const int total = n * TC;
-                for (int e = tid; e < total; e += kThreads) {
-                    const int i = e / TC, k = e - i * TC;
-                    if (c0 + k < d)
-                        cp_async4(sbase + (uint32_t)e * 4u, copies + (int64_t)rows[i] * ld + c0 + k);
-                }
-            }
-        }
-        cp_async_commit();
-    };
-
-    const int64_t t0 = blockIdx.x;
-    if constexpr (STAGES == 1) {
-        issue(t0, 0);
-    } else {
-#pragma unroll
-        for (int q = 0; q < STAGES - 1; ++q) issue(t0 + (int64_t)q * gridDim.x, q);
-    }
-
-    // Bin search over the 128 bins of the coordinates whose threads pass hm:
-    // slot u sums bins [u*BPT, u*BPT + BPT) over the coordinate's SUB
-    // columns; the slot holding rank `rank` resolves the bin and writes
-    // S_BIN, S_REM (rank inside the bin) and S_CNT.  Leaves the histogram
-    // zeroed.  Called by every thread (two block barriers).
-    auto bin_search = [&](bool hm, uint32_t rank) {
-        uint32_t cb[BPT];
-        uint32_t sum = 0u;
-#pragma unroll
-        for (int j = 0; j < BPT; ++j) {
-            uint32_t v = 0u;
-            if (hm) {
-                const int b = slot * BPT + j;
-#pragma unroll
-                for (int s2 = 0; s2 < SUB; ++s2) v += hist[b * 32 + s2 * TC + c];
-            }
-            cb[j] = v;
-            sum += v;
-        }
-        if (hm) part[slot * TC + c] = sum;
-        __syncthreads();
-        for (int i = tid * 4; i < kNB * 32; i += kThreads * 4)
-            *reinterpret_cast<uint4 *>(hist + i) = make_uint4(0u, 0u, 0u, 0u);
-        if (hm) {
-            uint32_t rem = rank;
-            int owner = NS - 1;
-            bool fd = false;
-            for (int u = 0; u < NS; ++u) {
-                const uint32_t pu = part[u * TC + c];
-                const bool hit = !fd && rem < pu;
-                if (hit) owner = u;
-                if (!fd && !hit) rem -= pu;
-                fd |= hit;
-            }
-            if (owner == slot) {
-                uint32_t bsel = BPT - 1, csel = cb[BPT - 1];
-                bool f2 = false;
-#pragma unroll
-                for (int j = 0; j < BPT; ++j) {
-                    const bool hit = !f2 && rem < cb[j];
-                    if (hit) {
-                        bsel = (uint32_t)j;
-                        csel = cb[j];
+                for (uint32_t e = 0; e < cnt; ++e) {
+                    const uint32_t x = to_key(list[e * TC + c]);
+                    uint32_t lt = 0u, le = 0u;
+                    for (uint32_t t2 = 0; t2 < cnt; ++t2) {
+                        const uint32_t y = to_key(list[t2 * TC + c]);
+                        lt += y < x;
+                        le += y <= x;
                     }
-                    if (!f2 && !hit) rem -= cb[j];
-                    f2 |= hit;
+                    if (lt <= rk && rk < le) res = x;
                 }
-                S(S_BIN) = (uint32_t)(slot * BPT) + bsel;
-                S(S_REM) = rem;
-                S(S_CNT) = csel;
             }
-        }
-        __syncthreads();
-    };
-
-    // rank the cnt keys of the coordinate's list; the candidate(s) of rank
-    // `rank` write the output
-    auto rank_list = [&](bool act, uint32_t cnt, uint32_t rank, int64_t oc) {
-        if (!act) return;
-        for (uint32_t e = (uint32_t)slot; e < cnt; e += NS) {
-            const uint32_t x = list[e * TC + c];
-            uint32_t lt = 0u, le = 0u;
-            for (uint32_t t2 = 0; t2 < cnt; ++t2) {
-                const uint32_t y = list[t2 * TC + c];
-                lt += y < x;
-                le += y <= x;
-            }
-            if (lt <= rank && rank < le) out[oc] = __uint_as_float(from_key(x));
+            out[c0_p + c] = __uint_as_float(from_key(res));
         }
     };
 
-    int stage = 0;
-    for (int64_t t = t0; t < ntiles; t += gridDim.x) {
-        if constexpr (STAGES > 1)
-            issue(t + (int64_t)(STAGES - 1) * gridDim.x, (stage + STAGES - 1) % STAGES);
-        bool fetched = false;
-        cp_async_wait<STAGES - 1>();
-        __syncthreads();
-        const uint32_t *tile = reinterpret_cast<const uint32_t *>(tiles + stage * L.tile_bytes);
+    for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x) {
         const int64_t c0 = t * TC;
-        const int64_t oc = c0 + c;
-        const bool live = oc < d;
-        const uint32_t *pv = tile + slot * TC + c;       // value j of this slot: pv[j * VS]
+        const bool lv = c0 + lane * V < d;                 // some coordinate of the lane is live
+        const char *lb = lane_base(t);
+        const int64_t tn = t + gridDim.x;
+        const bool lvn = tn < ntiles && tn * TC + lane * V < d;
+        const char *lbn = lvn ? lane_base(tn) : lb;
+
+        // One pass over this warp's rows, batch by batch: fn(x, j, u) for
+        // every row; each register is refilled right after it is used.
+        auto sweep = [&](auto fn) {
+            auto batch = [&](auto lastc, int j0) {
+                constexpr bool LAST = decltype(lastc)::value;
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    if constexpr (LAST) {
+                        if (j0 + u < nmine) fn(xa[u], j0 + u, u);
+                        xa[u] = (lvn && u < nmine) ? load_row<V>(row_ptr(lbn, u)) : T{};
+                    } else {
+                        fn(xa[u], j0 + u, u);
+                        const int jn = j0 + kU + u;
+                        xa[u] = (lv && jn < nmine) ? load_row<V>(row_ptr(lb, jn)) : T{};
+                    }
+                }
+            };
+            int j0 = 0;
+            for (; j0 + kU < nmine; j0 += kU) batch(std::false_type{}, j0);
+            batch(std::true_type{}, j0);
+        };
 
         if constexpr (MODE == 1) {
-            // ---- mean: compensated per-slot sums, combined in slot order
-            float sm = 0.f, e = 0.f;
-            for (int j = 0; j < nmine; ++j) {
-                float ns, ne;
-                two_sum(sm, __uint_as_float(pv[j * VS]), ns, ne);
-                sm = ns;
-                e += ne;
-            }
-            part[slot * TC + c] = __float_as_uint(sm);
-            part[(NS + slot) * TC + c] = __float_as_uint(e);
-            __syncthreads();
-            if (slot == 0 && live) {
-                float a = 0.f, ae = 0.f;
-                for (int u = 0; u < NS; ++u) {
+            // ---- mean: compensated per-thread sums, combined in warp order
+            float sm[V], se[V];
+#pragma unroll
+            for (int k = 0; k < V; ++k) sm[k] = se[k] = 0.f;
+            sweep([&](const T &x, int, int) {
+#pragma unroll
+                for (int k = 0; k < V; ++k) {
                     float ns, ne;
-                    two_sum(a, __uint_as_float(part[u * TC + c]), ns, ne);
-                    a = ns;
-                    ae += ne + __uint_as_float(part[(NS + u) * TC + c]);
+                    two_sum(sm[k], __uint_as_float(elem<V>(x, k)), ns, ne);
+                    sm[k] = ns;
+                    se[k] += ne;
                 }
-                out[oc] = (float)(((double)a + (double)ae) / (double)n);
+            });
+#pragma unroll
+            for (int k = 0; k < V; ++k) {
+                list[(2 * w) * TC + lane * V + k] = __float_as_uint(sm[k]);
+                list[(2 * w + 1) * TC + lane * V + k] = __float_as_uint(se[k]);
             }
+            __syncthreads();
+            for (int c = tid; c < TC; c += kThreads) {
+                if (c0 + c >= d) continue;
+                float a = 0.f, ae = 0.f;
+                for (int u = 0; u < kWarps; ++u) {
+                    float ns, ne;
+                    two_sum(a, __uint_as_float(list[(2 * u) * TC + c]), ns, ne);
+                    a = ns;
+                    ae += ne + __uint_as_float(list[(2 * u + 1) * TC + c]);
+                }
+                out[c0 + c] = (float)(((double)a + (double)ae) / (double)n);
+            }
+            __syncthreads();
         } else {
-            uint32_t *tw = tags + slot * TC + c;         // tag word q of this slot: tw[q * VS]
-
-            // ---- S: sample key range
-            uint32_t klo = 0xffffffffu, khi = 0u;
-            if (live && nmine > 0) {
-                const uint32_t k = to_key(pv[0]);
-                klo = min(klo, k);
-                khi = max(khi, k);
+            // ---- S: key range of the sample (rows 0 and 1 of every warp)
+            if (lv) {
+#pragma unroll
+                for (int k = 0; k < V; ++k) {
+                    if (c0 + lane * V + k >= d) continue;
+                    uint32_t lo = 0xffffffffu, hi = 0u;
+                    if (nmine > 0) {
+                        const uint32_t q = to_key(elem<V>(xa[0], k));
+                        lo = min(lo, q);
+                        hi = max(hi, q);
+                    }
+                    if (nmine > 1) {
+                        const uint32_t q = to_key(elem<V>(xa[1], k));
+                        lo = min(lo, q);
+                        hi = max(hi, q);
+                    }
+                    if (lo <= hi) {
+                        atomicMin(&S(S_MIN, lane * V + k), lo);
+                        atomicMax(&S(S_MAX, lane * V + k), hi);
+                    }
+                }
             }
-            if (live && nmine > 1) {
-                const uint32_t k = to_key(pv[VS]);
-                klo = min(klo, k);
-                khi = max(khi, k);
+            __syncthreads();                                        // (B)
+            float vs[V], vc[V];
+            uint32_t hb[NP];
+#pragma unroll
+            for (int k = 0; k < V; ++k) {
+                const float xlo = __uint_as_float(from_key(S(S_MIN, lane * V + k)));
+                const float xhi = __uint_as_float(from_key(S(S_MAX, lane * V + k)));
+                // sample range -> y in [1/126, 125/126]: bins 1..125
+                const float sc = (124.0f / 126.0f) / (xhi - xlo);
+                const float cc = fmaf(-xlo, sc, 1.0f / 126.0f);
+                const bool ok = isfinite(xlo) && isfinite(xhi) && xhi > xlo && isfinite(sc) &&
+                                sc > 0.f && isfinite(cc);
+                vs[k] = ok ? sc : 0.f;
+                vc[k] = ok ? cc : 0.f;
+                if (w == 0) {
+                    const bool live = c0 + lane * V + k < d;
+                    S(S_MODE, lane * V + k) = !live ? M_DONE : (ok ? M_VH : M_KA);
+                }
             }
 #pragma unroll
-            for (int o = TC; o < 32; o <<= 1) {
-                klo = min(klo, __shfl_xor_sync(full, klo, o));
-                khi = max(khi, __shfl_xor_sync(full, khi, o));
-            }
-            if (s == 0 && live) {
-                atomicMin(&S(S_SMIN), klo);
-                atomicMax(&S(S_SMAX), khi);
-            }
-            __syncthreads();
-            const float xs_lo = __uint_as_float(from_key(S(S_SMIN)));
-            const float xs_hi = __uint_as_float(from_key(S(S_SMAX)));
-            const float vs = (float)(kNB - 2) / (xs_hi - xs_lo);
-            const float vc = 8388609.0f - xs_lo * vs;    // xs_lo -> about 2^23 + 1
-            const bool vspace = isfinite(xs_lo) && isfinite(xs_hi) && xs_hi > xs_lo &&
-                                isfinite(vs) && isfinite(vc);
-            int mode = !live ? M_DONE : (vspace ? M_VH : M_KA);
+            for (int p = 0; p < NP; ++p)
+                hb[p] = hist_s + (uint32_t)(p * 32 + lane) * 4u - (0x4B000000u << SHB);
 
-            // ---- VH: histogram of every value, tags, NaN check
-            if (mode == M_VH) {
-                uint32_t *hl = hist + lane;
-                float nacc = 0.f;
-                const uint32_t *p = pv;
-                uint32_t *q4 = tw;
-                int j = 0;
-#pragma unroll 2
-                for (; j + 4 <= nmine; j += 4, p += 4 * VS, q4 += VS) {
-                    const float y0 = fmaf(__uint_as_float(p[0]), vs, vc);
-                    const float y1 = fmaf(__uint_as_float(p[VS]), vs, vc);
-                    const float y2 = fmaf(__uint_as_float(p[2 * VS]), vs, vc);
-                    const float y3 = fmaf(__uint_as_float(p[3 * VS]), vs, vc);
-                    nacc = max_nan(max_nan(nacc, max_nan(y0, y1)), max_nan(y2, y3));
-                    const uint32_t b0 = vbin(y0), b1 = vbin(y1), b2 = vbin(y2), b3 = vbin(y3);
-                    atomicAdd(hl + b0 * 32, 1u);
-                    atomicAdd(hl + b1 * 32, 1u);
-                    atomicAdd(hl + b2 * 32, 1u);
-                    atomicAdd(hl + b3 * 32, 1u);
-                    *q4 = pack4(b0, b1, b2, b3);
+            // ---- sweep: the pending tile's members (old tag words), then
+            // VH for this tile (histogram, new tag words, NaN check)
+            uint32_t nanf = 0u, tacc = 0u;
+            sweep([&](const T &x, int j, int u) {
+                if (u % RPW == 0) {
+                    const uint32_t z = tag_match(tags[((j / RPW) * kWarps + w) * 32 + lane], vbx_p);
+                    if (z) capture(z, j / RPW);
                 }
-                if (j < nmine) {
-                    // last, partial word: missing rows get tag 0xFF, which no bin has
-                    uint32_t word = 0xFFFFFFFFu;
-                    for (int k = 0; j < nmine; ++j, ++k, p += VS) {
-                        const float y = fmaf(__uint_as_float(*p), vs, vc);
-                        nacc = max_nan(nacc, y);
-                        const uint32_t b = vbin(y);
-                        atomicAdd(hl + b * 32, 1u);
-                        word = (word & ~(0xFFu << (8 * k))) | (b << (8 * k));
+                uint32_t bb[V];
+#pragma unroll
+                for (int k = 0; k < V; ++k) {
+                    bb[k] = vbin_bits(__uint_as_float(elem<V>(x, k)), vs[k], vc[k]);
+                    const uint32_t a = (bb[k] << SHB) + hb[k / 2];
+                    if (k & 1) red_shared<0x10000u>(a);
+                    else red_shared<1u>(a);
+                }
+                if constexpr (V == 4) {
+                    nan_check(nanf, __uint_as_float(x.x), __uint_as_float(x.y),
+                              __uint_as_float(x.z), __uint_as_float(x.w));
+                    tags[(j * kWarps + w) * 32 + lane] = pack4(bb[0], bb[1], bb[2], bb[3]);
+                } else if constexpr (V == 2) {
+                    nan_check(nanf, __uint_as_float(x.x), __uint_as_float(x.y),
+                              __uint_as_float(x.x), __uint_as_float(x.y));
+                    const uint32_t h = __byte_perm(bb[0], bb[1], 0x0040) & 0xFFFFu;
+                    if ((u & 1) == 0) {
+                        tacc = h | (kPadTag * 0x01010000u);
+                        if (j + 1 >= nmine) tags[((j >> 1) * kWarps + w) * 32 + lane] = tacc;
+                    } else {
+                        tags[((j >> 1) * kWarps + w) * 32 + lane] = (tacc & 0xFFFFu) | (h << 16);
                     }
-                    *q4 = word;
+                } else {
+                    nan_check(nanf, __uint_as_float(x), __uint_as_float(x),
+                              __uint_as_float(x), __uint_as_float(x));
+                    const int sh = 8 * (u & 3);
+                    tacc = ((u & 3) == 0 ? kPadTag * 0x01010101u : tacc);
+                    tacc = (tacc & ~(0xFFu << sh)) | ((bb[0] & 0xFFu) << sh);
+                    if ((u & 3) == 3 || j + 1 >= nmine) tags[((j >> 2) * kWarps + w) * 32 + lane] = tacc;
                 }
-                if (nacc != nacc) atomicOr(&S(S_NAN), 1u);
+            });
+            cp_async_commit();
+            if (nanf) {
+#pragma unroll
+                for (int k = 0; k < V; ++k) atomicOr(&S(S_NAN, lane * V + k), 1u);
             }
-            __syncthreads();
-            if (mode == M_VH && S(S_NAN) != 0u) mode = M_KA;     // exact key-space passes
-            if (slot == 0) {
-                S(S_SMIN) = 0xffffffffu;
-                S(S_SMAX) = 0u;
-            }
-
-            // ---- B: the bin holding the median
-            bin_search(mode == M_VH, krank);
-            uint32_t vb = 0u, krem = krank, cnt = (uint32_t)n;
-            if (mode == M_VH) {
-                vb = S(S_BIN);
-                krem = S(S_REM);
-                cnt = S(S_CNT);
-                mode = cnt <= (uint32_t)kCap ? M_VC : M_VM;
-            }
-            if (slot == 0) S(S_NAN) = 0u;
-
-            // ---- VC: list the members of bin vb
-            if (mode == M_VC) {
-                const uint32_t vbx = vb * 0x01010101u;
-                const int nw = (nmine + 3) >> 2;
-                uint32_t wm = 0u;                     // words holding a member (first 32)
-                for (int q = 0; q < nw && q < 32; ++q)
-                    wm |= (tag_match(tw[q * VS], vbx) != 0u ? 1u : 0u) << q;
-                for (; wm; wm &= wm - 1u) {
-                    const int q = __ffs(wm) - 1;
-                    uint32_t z = tag_match(tw[q * VS], vbx);
-                    uint32_t pos = atomicAdd(&S(S_LCNT), (uint32_t)__popc(z));
-                    for (; z && pos < (uint32_t)kCap; z &= z - 1u)
-                        list[(pos++) * TC + c] = to_key(pv[(q * 4 + ((__ffs(z) - 1) >> 3)) * VS]);
+            cp_async_wait_all();
+            __syncthreads();                                        // (C)
+            if (have_p) rank_pending();
+            if (w == 0) {
+#pragma unroll
+                for (int k = 0; k < V; ++k) {
+                    const int c = lane * V + k;
+                    if (S(S_MODE, c) == M_VH && S(S_NAN, c)) S(S_MODE, c) = M_KA;
+                    S(S_NAN, c) = 0u;
+                    S(S_MIN, c) = 0xffffffffu;
+                    S(S_MAX, c) = 0u;
                 }
-                for (int q = 32; q < nw; ++q) {       // slots with more than 128 rows
-                    uint32_t z = tag_match(tw[q * VS], vbx);
-                    if (z) {
-                        uint32_t pos = atomicAdd(&S(S_LCNT), (uint32_t)__popc(z));
-                        for (; z && pos < (uint32_t)kCap; z &= z - 1u)
-                            list[(pos++) * TC + c] = to_key(pv[(q * 4 + ((__ffs(z) - 1) >> 3)) * VS]);
+            }
+            __syncthreads();                                        // (R)
+            for (int c = tid; c < TC; c += kThreads) S(S_LCNT, c) = 0u;
+
+            // ---- B1: per-warp partial sums over bins [16w, 16w + 16)
+            {
+                uint32_t ps[NP];
+#pragma unroll
+                for (int p = 0; p < NP; ++p) ps[p] = 0u;
+#pragma unroll
+                for (int b = 0; b < 16; ++b)
+#pragma unroll
+                    for (int p = 0; p < NP; ++p) ps[p] += hist[((w * 16 + b) * NP + p) * 32 + lane];
+#pragma unroll
+                for (int k = 0; k < V; ++k)
+                    list[w * TC + lane * V + k] = (ps[k / 2] >> (16 * (k & 1))) & 0xFFFFu;
+            }
+            __syncthreads();                                        // (D)
+            // ---- B2: one thread per coordinate resolves its bin
+            for (int c = tid; c < TC; c += kThreads) {
+                uint32_t pc = 0u;
+                if (S(S_MODE, c) == M_VH) {
+                    uint32_t rem = krank;
+                    int owner = kWarps - 1;
+                    bool fd = false;
+                    for (int u = 0; u < kWarps; ++u) {
+                        const uint32_t pu = list[u * TC + c];
+                        const bool hit = !fd && rem < pu;
+                        if (hit) owner = u;
+                        if (!fd && !hit) rem -= pu;
+                        fd |= hit;
                     }
+                    const int lc = c / V, k = c % V;
+                    const uint32_t *h = hist + (k / 2) * 32 + lc;
+                    const int shf = 16 * (k & 1);
+                    int bin = owner * 16 + 15;
+                    uint32_t cnt = 0u;
+                    bool f2 = false;
+                    for (int b = owner * 16; b < owner * 16 + 16; ++b) {
+                        const uint32_t cb = (h[b * NP * 32] >> shf) & 0xFFFFu;
+                        const bool hit = !f2 && rem < cb;
+                        if (hit) {
+                            bin = b;
+                            cnt = cb;
+                        }
+                        if (!f2 && !hit) rem -= cb;
+                        f2 |= hit;
+                    }
+                    S(S_BIN, c) = (uint32_t)bin;
+                    S(S_REM, c) = rem;
+                    S(S_CNT, c) = cnt;
+                    S(S_PREM, c) = rem;
+                    const bool vcm = cnt <= (uint32_t)kCap;
+                    S(S_MODE, c) = vcm ? M_VC : M_VM;
+                    pc = vcm ? cnt : 0u;
                 }
+                S(S_PCNT, c) = pc;
             }
-            const bool general = __syncthreads_or(mode != M_DONE && mode != M_VC);
-            if (slot == 0) S(S_LCNT) = 0u;
-            if constexpr (STAGES == 1) {
-                if (!general) {
-                    issue(t + gridDim.x, 0);          // the tile is no longer read
-                    fetched = true;
-                }
-            }
-            rank_list(mode == M_VC, cnt, krem, oc);
-            if (mode == M_VC) mode = M_DONE;
+            __syncthreads();                                        // (E)
+            for (int i = tid * 4; i < kNB * NP * 32; i += kThreads * 4)
+                *reinterpret_cast<uint4 *>(hist + i) = make_uint4(0u, 0u, 0u, 0u);
 
-            if (general) {
-                // ---- exact fallback passes (rare)
-                uint32_t lo = 0u, hi = 0u;
+            // this tile becomes the pending one: target bins of its coordinates
+            uint32_t vbx = 0u, vcm = 0u;
+            bool need_general = false;
+#pragma unroll
+            for (int k = 0; k < V; ++k) {
+                const uint32_t md = S(S_MODE, lane * V + k);
+                const uint32_t vb = md == M_VC ? S(S_BIN, lane * V + k) : 0xFFu;
+                vcm |= (md == M_VC ? 1u : 0u) << k;
+                need_general |= md == M_VM || md == M_KA;
+#pragma unroll
+                for (int q = k; q < 4; q += V) vbx |= vb << (8 * q);
+            }
+            have_p = true;
+            lb_p = lb;
+            c0_p = c0;
+            vbx_p = vbx;
+            vcm_p = vcm;
+
+            if (__syncthreads_or(need_general)) {
+                // ---- exact fallback passes (rare), values re-read from global memory
+                auto reread = [&](int j, int k) -> uint32_t {
+                    return __ldcg(reinterpret_cast<const unsigned int *>(row_ptr(lb, j)) + k);
+                };
                 for (int it = 0; it < kMaxPasses; ++it) {
-                    const int m0 = mode;
-                    const uint32_t W = hi - lo;
-                    const int bits = 32 - __clz(W);
-                    const int sh = bits > kLogNB ? bits - kLogNB : 0;
-                    if (m0 == M_VM || m0 == M_KA) {
-                        uint32_t a = 0xffffffffu, b = 0u;
-                        const uint8_t *tb = reinterpret_cast<const uint8_t *>(tw);
-                        for (int j = 0; j < nmine; ++j) {
-                            const bool take = m0 == M_KA || tb[(j >> 2) * VS * 4 + (j & 3)] == vb;
-                            if (take) {
-                                const uint32_t k = to_key(pv[j * VS]);
-                                a = min(a, k);
-                                b = max(b, k);
+                    // pass over the values of the coordinates still searching
+                    if (lv) {
+                        for (int k = 0; k < V; ++k) {
+                            const int c = lane * V + k;
+                            const uint32_t md = S(S_MODE, c);
+                            if (md == M_DONE || md == M_VC) continue;
+                            const uint32_t lo = S(S_LO, c), hi = S(S_HI, c);
+                            const uint32_t W = hi - lo;
+                            const int bits = 32 - __clz(W);
+                            const int sh = bits > kLogNB ? bits - kLogNB : 0;
+                            const uint32_t vb = S(S_BIN, c);
+                            const uint8_t *tb = reinterpret_cast<const uint8_t *>(tags);
+                            uint32_t a = 0xffffffffu, bmax = 0u;
+                            for (int j = 0; j < nmine; ++j) {
+                                if (md == M_VM) {
+                                    const int q = j / RPW, p = (j % RPW) * V + k;
+                                    if (tb[((q * kWarps + w) * 32 + lane) * 4 + p] != vb) continue;
+                                }
+                                const uint32_t key = to_key(reread(j, k));
+                                if (md == M_VM || md == M_KA) {
+                                    a = min(a, key);
+                                    bmax = max(bmax, key);
+                                } else if (key - lo <= W) {
+                                    if (md == M_KH) {
+                                        atomicAdd(hist + (((key - lo) >> sh) * NP + k / 2) * 32 + lane,
+                                                  (k & 1) ? 0x10000u : 1u);
+                                    } else {
+                                        const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
+                                        if (at < (uint32_t)kCap) list[at * TC + c] = key;
+                                    }
+                                }
                             }
-                        }
-                        if (a <= b) {
-                            atomicMin(&S(S_KMIN), a);
-                            atomicMax(&S(S_KMAX), b);
-                        }
-                    } else if (m0 == M_KH) {
-                        for (int j = 0; j < nmine; ++j) {
-                            const uint32_t dk = to_key(pv[j * VS]) - lo;
-                            if (dk <= W) atomicAdd(hist + (dk >> sh) * 32 + lane, 1u);
-                        }
-                    } else if (m0 == M_KC) {
-                        for (int j = 0; j < nmine; ++j) {
-                            const uint32_t k = to_key(pv[j * VS]);
-                            if (k - lo <= W) {
-                                const uint32_t pos = atomicAdd(&S(S_LCNT), 1u);
-                                if (pos < (uint32_t)kCap) list[pos * TC + c] = k;
+                            if ((md == M_VM || md == M_KA) && a <= bmax) {
+                                atomicMin(&S(S_MIN, c), a);
+                                atomicMax(&S(S_MAX, c), bmax);
                             }
                         }
                     }
                     __syncthreads();
-                    if (m0 == M_VM || m0 == M_KA) {
-                        lo = S(S_KMIN);
-                        hi = S(S_KMAX);
-                        if (m0 == M_KA) {
-                            krem = krank;
-                            cnt = (uint32_t)n;
-                        }
-                        if (lo == hi) {
-                            if (slot == 0) out[oc] = __uint_as_float(from_key(lo));
-                            mode = M_DONE;
-                        } else {
-                            mode = cnt <= (uint32_t)kCap ? M_KC : M_KH;
-                        }
-                    }
-                    rank_list(m0 == M_KC, cnt, krem, oc);
-                    if (m0 == M_KC) mode = M_DONE;
-                    if (__syncthreads_or(m0 == M_KH)) {
-                        bin_search(m0 == M_KH, krem);
-                        if (m0 == M_KH) {
-                            const uint32_t nb = S(S_BIN);
-                            krem = S(S_REM);
-                            cnt = S(S_CNT);
-                            const uint32_t nlo = lo + (nb << sh);
+                    // resolution, one thread per coordinate
+                    for (int c = tid; c < TC; c += kThreads) {
+                        const uint32_t md = S(S_MODE, c);
+                        if (md == M_DONE || md == M_VC) continue;
+                        uint32_t lo = S(S_LO, c), hi = S(S_HI, c);
+                        uint32_t rk = S(S_REM, c), cnt = S(S_CNT, c);
+                        uint32_t nm = md;
+                        if (md == M_VM || md == M_KA) {
+                            lo = S(S_MIN, c);
+                            hi = S(S_MAX, c);
+                            if (md == M_KA) {
+                                rk = krank;
+                                cnt = (uint32_t)n;
+                            }
+                            nm = lo == hi ? M_DONE : (cnt <= (uint32_t)kCap ? M_KC : M_KH);
+                        } else if (md == M_KH) {
+                            const uint32_t W = hi - lo;
+                            const int bits = 32 - __clz(W);
+                            const int sh = bits > kLogNB ? bits - kLogNB : 0;
+                            const int lc = c / V, k = c % V;
+                            const uint32_t *h = hist + (k / 2) * 32 + lc;
+                            const int shf = 16 * (k & 1);
+                            uint32_t b = 0;
+                            for (; b < (uint32_t)kNB - 1; ++b) {
+                                const uint32_t cb = (h[b * NP * 32] >> shf) & 0xFFFFu;
+                                if (rk < cb) break;
+                                rk -= cb;
+                            }
+                            cnt = (h[b * NP * 32] >> shf) & 0xFFFFu;
+                            const uint32_t nlo = lo + (b << sh);
                             const uint64_t top = (uint64_t)nlo + ((1ull << sh) - 1ull);
                             hi = top < (uint64_t)hi ? (uint32_t)top : hi;
                             lo = nlo;
-                            if (lo == hi) {
-                                if (slot == 0) out[oc] = __uint_as_float(from_key(lo));
-                                mode = M_DONE;
-                            } else {
-                                mode = cnt <= (uint32_t)kCap ? M_KC : M_KH;
+                            nm = lo == hi ? M_DONE : (cnt <= (uint32_t)kCap ? M_KC : M_KH);
+                        } else if (md == M_KC) {
+                            const uint32_t m = min(cnt, (uint32_t)kCap);
+                            for (uint32_t e = 0; e < m; ++e) {
+                                const uint32_t x = list[e * TC + c];
+                                uint32_t lt = 0u, le = 0u;
+                                for (uint32_t t2 = 0; t2 < m; ++t2) {
+                                    const uint32_t y = list[t2 * TC + c];
+                                    lt += y < x;
+                                    le += y <= x;
+                                }
+                                if (lt <= rk && rk < le) {
+                                    lo = x;
+                                    break;
+                                }
                             }
+                            hi = lo;
+                            nm = M_DONE;
                         }
+                        if (nm == M_DONE) out[c0 + c] = __uint_as_float(from_key(lo));
+                        S(S_LO, c) = lo;
+                        S(S_HI, c) = hi;
+                        S(S_REM, c) = rk;
+                        S(S_CNT, c) = cnt;
+                        S(S_MODE, c) = nm;
+                        S(S_MIN, c) = 0xffffffffu;
+                        S(S_MAX, c) = 0u;
+                        S(S_LCNT, c) = 0u;
                     }
-                    if (slot == 0) {
-                        S(S_KMIN) = 0xffffffffu;
-                        S(S_KMAX) = 0u;
-                        S(S_LCNT) = 0u;
+                    __syncthreads();
+                    for (int i = tid * 4; i < kNB * NP * 32; i += kThreads * 4)
+                        *reinterpret_cast<uint4 *>(hist + i) = make_uint4(0u, 0u, 0u, 0u);
+                    bool more = false;
+                    for (int c = tid; c < TC; c += kThreads) {
+                        const uint32_t md = S(S_MODE, c);
+                        more |= md != M_DONE && md != M_VC;
                     }
-                    if (!__syncthreads_or(mode != M_DONE)) break;
+                    if (!__syncthreads_or(more)) break;
                 }
             }
         }
-        if (!fetched) {
-            __syncthreads();
-            if constexpr (STAGES == 1) issue(t + gridDim.x, 0);
-        }
-        stage = (stage + 1) % STAGES;
     }
-    cp_async_wait<0>();
+    if constexpr (MODE == 0) {
+        // the last tile's members: scan its tags, then rank
+        if (have_p) {
+            for (int q = 0; q < nwords; ++q) {
+                const uint32_t z = tag_match(tags[(q * kWarps + w) * 32 + lane], vbx_p);
+                if (z) capture(z, q);
+            }
+            cp_async_commit();
+            cp_async_wait_all();
+            __syncthreads();
+            rank_pending();
+        }
+    }
 }
 
 size_t smem_cap()
@@ -548,15 +676,15 @@ size_t smem_cap()
     return (size_t)cap - 1024;        // static shared memory and reserve
 }
 
-template <int TC, int STAGES, int MINB, bool VEC, int MODE>
+template <int V, int MINB, bool W32, int MODE>
 cudaError_t try_launch(bool &launched, const float *copies, int64_t f, int r, int64_t d,
                        int64_t ld, const int8_t *sel, aspis_detection *det, float *out,
                        cudaStream_t stream)
 {
     launched = false;
-    const Layout L = make_layout<TC, STAGES>(f);
+    const Layout L = make_layout<V>(f);
     if (L.total > smem_cap()) return cudaSuccess;
-    auto kern = aggregate_kernel<TC, STAGES, MINB, VEC, MODE>;
+    auto kern = aggregate_kernel<V, MINB, W32, MODE>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)L.total);
     if (e != cudaSuccess) return e;
@@ -564,7 +692,7 @@ cudaError_t try_launch(bool &launched, const float *copies, int64_t f, int r, in
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, L.total);
     if (e != cudaSuccess) return e;
     if (per_sm < MINB) return cudaSuccess;        // the next configuration is tried
-    const int64_t ntiles = (d + TC - 1) / TC;
+    const int64_t ntiles = (d + Geo<V>::TC - 1) / Geo<V>::TC;
     int64_t grid = (int64_t)sm_count() * per_sm;
     if (grid > ntiles) grid = ntiles;
     kern<<<(unsigned)grid, kThreads, L.total, stream>>>(copies, f, r, d, ld, sel, det, out);
@@ -572,25 +700,29 @@ cudaError_t try_launch(bool &launched, const float *copies, int64_t f, int r, in
     return cudaGetLastError();
 }
 
-template <bool VEC, int MODE>
-cudaError_t launch_mode(const float *copies, int64_t f, int r, int64_t d, int64_t ld,
+template <int MODE, bool W32>
+cudaError_t launch_mode(int align, const float *copies, int64_t f, int r, int64_t d, int64_t ld,
                         const int8_t *sel, aspis_detection *det, float *out, cudaStream_t stream)
 {
     bool ok = false;
     cudaError_t e = cudaSuccess;
-#define ASPIS_TRY(TC, ST, MB)                                                                  \
-    e = try_launch<TC, ST, MB, VEC, MODE>(ok, copies, f, r, d, ld, sel, det, out, stream);     \
+#define ASPIS_TRY(V, MB)                                                                        \
+    e = try_launch<V, MB, W32, MODE>(ok, copies, f, r, d, ld, sel, det, out, stream);           \
     if (e != cudaSuccess || ok) return e;
-    if constexpr (VEC) {
-        ASPIS_TRY(32, 1, 2)
-        ASPIS_TRY(32, 2, 1)
-        ASPIS_TRY(16, 1, 2)
-        ASPIS_TRY(16, 2, 1)
-        ASPIS_TRY(8, 1, 2)
-        ASPIS_TRY(8, 2, 1)
-        ASPIS_TRY(8, 1, 1)
+    if (align >= 4) {
+        ASPIS_TRY(4, 2)
     }
-    ASPIS_TRY(4, 1, 1)
+    if (align >= 2) {
+        ASPIS_TRY(2, 2)
+    }
+    if (align >= 4) {
+        ASPIS_TRY(4, 1)
+    }
+    if (align >= 2) {
+        ASPIS_TRY(2, 1)
+    }
+    ASPIS_TRY(1, 2)
+    ASPIS_TRY(1, 1)
 #undef ASPIS_TRY
     return cudaErrorInvalidValue;
 }
@@ -601,13 +733,16 @@ cudaError_t launch_aggregate(const float *copies, int64_t f, int r, int64_t d, i
                              const int8_t *sel, aspis_detection *det, int mode, float *out,
                              cudaStream_t stream)
 {
-    if (f > ASPIS_MAX_AGG_FILES) return cudaErrorInvalidValue;
-    const bool vec = ((uintptr_t)copies % 16 == 0) && (ld % 4 == 0);
-    if (vec)
-        return mode == 0 ? launch_mode<true, 0>(copies, f, r, d, ld, sel, det, out, stream)
-                         : launch_mode<true, 1>(copies, f, r, d, ld, sel, det, out, stream);
-    return mode == 0 ? launch_mode<false, 0>(copies, f, r, d, ld, sel, det, out, stream)
-                     : launch_mode<false, 1>(copies, f, r, d, ld, sel, det, out, stream);
+    if (f > ASPIS_MAX_AGG_FILES || f * r > 65535) return cudaErrorInvalidValue;
+    // widest load every row start allows: 16 bytes (V = 4), 8 (V = 2), else 4
+    const uintptr_t p = (uintptr_t)copies;
+    const int align = (p % 16 == 0 && ld % 4 == 0) ? 4 : (p % 8 == 0 && ld % 2 == 0) ? 2 : 1;
+    const bool w32 = (uint64_t)ld * 4u < (1ull << 32);     // row pitch fits a 32-bit multiplier
+    if (mode == 0)
+        return w32 ? launch_mode<0, true>(align, copies, f, r, d, ld, sel, det, out, stream)
+                   : launch_mode<0, false>(align, copies, f, r, d, ld, sel, det, out, stream);
+    return w32 ? launch_mode<1, true>(align, copies, f, r, d, ld, sel, det, out, stream)
+               : launch_mode<1, false>(align, copies, f, r, d, ld, sel, det, out, stream);
 }
 
 }  // namespace aspis

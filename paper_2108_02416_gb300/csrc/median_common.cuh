@@ -1,13 +1,16 @@
-// Pieces of the lower-median search (aggregate.cu): the totalOrder key map,
-// the value-space bin map, tag matching and the search modes.
+// Pieces of the coordinate-wise aggregation (aggregate.cu): the totalOrder
+// key map, the value-space bin map, tag matching, compensated sums and the
+// search modes of the lower median.
 #pragma once
 
 #include <stdint.h>
 
 namespace aspis {
 
-constexpr int kNB = 128;          // histogram bins per pass
+constexpr int kNB = 128;          // histogram rows (value-space bins use 0..126)
 constexpr int kLogNB = 7;
+constexpr int kTopBin = 126;      // value-space bins are 0..kTopBin
+constexpr uint32_t kPadTag = 0x7Fu;   // tag byte of a missing row: no value-space bin
 constexpr int kCap = 32;          // keys ranked directly
 
 // IEEE totalOrder as unsigned order: flip all bits of negatives, the sign
@@ -22,29 +25,31 @@ __device__ __forceinline__ uint32_t from_key(uint32_t k)
     return k ^ ((uint32_t)((int32_t)~k >> 31) | 0x80000000u);
 }
 
-// Value-space bin of y = fma(x, s, c): the integer part of y read from its
-// bits (y is near 2^23, where one unit is one ulp), clamped to [0, kNB).
-// The clamp is done on the float (an integer offset of a negative y's bits
-// would wrap), so negative y, -inf and underflow go to bin 0 and +inf or
-// large y to kNB-1.  Rounding is monotone, so the map is monotone in the IEEE
-// totalOrder of x for every non-NaN x.  NaNs are detected separately: fma
-// returns a canonical NaN whatever the sign of x (and it lands in bin 0).
-__device__ __forceinline__ uint32_t vbin(float y)
+// Value-space bin of x, as the bits of 2^23 + bin: y = sat(x*s + c) in
+// [0, 1] (fma with saturation: NaN gives +0), then 2^23 + rint(126*y), whose
+// low byte is the bin 0..126.  Both steps are correctly rounded and
+// non-decreasing, so the map is monotone in the IEEE totalOrder of every
+// non-NaN x (+0 and -0 share a bin) and always lands in 0..126, whatever s
+// and c are.  NaNs are detected separately.
+__device__ __forceinline__ uint32_t vbin_bits(float x, float s, float c)
 {
-    const float yc = fminf(fmaxf(y, 8388608.0f), 8388608.0f + (float)(kNB - 1));
-    return __float_as_uint(yc) - 0x4B000000u;
+    float y;
+    asm("fma.rn.sat.f32 %0, %1, %2, %3;" : "=f"(y) : "f"(x), "f"(s), "f"(c));
+    return __float_as_uint(fmaf(y, (float)kTopBin, 8388608.0f));
 }
 
-enum { M_DONE = 0, M_VH, M_VC, M_VM, M_VR, M_KA, M_KH, M_KC };
+enum { M_DONE = 0, M_VH, M_VC, M_VM, M_KA, M_KH, M_KC };
 
-// Four tag bytes against the replicated bin vbx: 0x80 in each byte whose tag
-// equals the bin.  Tags are < 0x80 and padding is 0xFF, so after the XOR a
-// byte is zero exactly at a match; OR-ing 0x80 first keeps the per-byte
-// subtraction from borrowing across bytes.
-__device__ __forceinline__ uint32_t tag_match(uint32_t word, uint32_t vbx)
+// Four tag bytes against the target bytes of vbx: 0x80 in each byte whose tag
+// equals its target.  Tags are < 0x80; a byte of w ^ vbx is then zero exactly
+// at a match, and for the other bytes OR-ing 0x80 keeps the per-byte
+// subtraction from borrowing across bytes.  Valid while no byte of w ^ vbx is
+// 0x80 (targets of coordinates that search nothing are 0xFF, which matches
+// only the padding tag 0x7F; callers skip such hits).
+__device__ __forceinline__ uint32_t tag_match(uint32_t w, uint32_t vbx)
 {
-    const uint32_t x = word ^ vbx;
-    return ~((x | 0x80808080u) - 0x01010101u) & ~x & 0x80808080u;
+    const uint32_t t = ((w ^ vbx) | 0x80808080u) - 0x01010101u;
+    return ~t & 0x80808080u;
 }
 
 // Two-sum: s + e == a + b exactly (Knuth); no products, so nothing to fuse.
