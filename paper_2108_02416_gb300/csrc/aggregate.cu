@@ -48,8 +48,9 @@
 namespace aspis {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 384;
 constexpr int kWarps = kThreads / 32;     // row slots of a CTA
+constexpr int kBPW = (kNB + kWarps - 1) / kWarps;   // histogram bins per warp in the bin search
 constexpr int kU = 8;                     // rows per load batch and thread
 constexpr int kMaxPasses = 12;            // fallback: VM/KA, at most 5 KH, KC
 
@@ -80,10 +81,12 @@ __device__ __forceinline__ typename Vec<V>::T load_row(const float *p)
     else return __ldcg(reinterpret_cast<const unsigned int *>(p));
 }
 
+// Histogram increment.  No memory clobber: the counters are read only after a
+// block barrier, so ordinary loads and stores may move across these.
 template <uint32_t INC>
 __device__ __forceinline__ void red_shared(uint32_t saddr)
 {
-    asm volatile("red.shared.add.u32 [%0], %1;\n" ::"r"(saddr), "n"(INC) : "memory");
+    asm volatile("red.shared.add.u32 [%0], %1;\n" ::"r"(saddr), "n"(INC));
 }
 
 __device__ __forceinline__ void cp_async4(uint32_t saddr, const void *g)
@@ -231,8 +234,10 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
         const int64_t t = blockIdx.x;
         const bool lv = t < ntiles && t * TC + lane * V < d;
 #pragma unroll
-        for (int u = 0; u < kU; ++u)
-            xa[u] = (lv && u < nmine) ? load_row<V>(row_ptr(lane_base(t), u)) : T{};
+        for (int u = 0; u < kU; ++u) {
+            xa[u] = T{};
+            if (lv && u < nmine) xa[u] = load_row<V>(row_ptr(lane_base(t), u));
+        }
     }
     __syncthreads();
 
@@ -243,19 +248,35 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     int64_t c0_p = 0;
     uint32_t vbx_p = 0xFFFFFFFFu, vcm_p = 0u;
 
-    // members of the pending tile among the four tag bytes of word q: their
-    // values are copied (4-byte cp.async) into the coordinate's list column
-    auto capture = [&](uint32_t z, int q) {
-        for (; z; z &= z - 1u) {
-            const int pos = (__ffs(z) - 1) >> 3;
-            const int j = q * RPW + pos / V, k = pos % V;
-            if (j < nmine && ((vcm_p >> k) & 1u)) {
-                const int c = lane * V + k;
-                const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
-                if (at < (uint32_t)kCap)
-                    cp_async4(list_s + (at * TC + c) * 4u, row_ptr(lb_p, j) + k);
+    // The members of the pending tile's bins: its tag words are compared with
+    // the target bins eight at a time (one mask bit per byte), and each
+    // member's value is copied (4-byte cp.async) into its coordinate's list
+    // column while the tile's rows are still in L2; the copies complete
+    // during the next sweep.
+    auto capture_members = [&]() {
+        if (!vcm_p) return;
+        for (int g = 0; g < nwords; g += 8) {
+            uint32_t m = 0u;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                if (g + i < nwords) {
+                    const uint32_t z = tag_match(tags[((g + i) * kWarps + w) * 32 + lane], vbx_p);
+                    m |= z >> (7 - i);
+                }
+            }
+            for (; m; m &= m - 1u) {
+                const int b = __ffs(m) - 1;
+                const int pos = b >> 3, q = g + (b & 7);
+                const int j = q * RPW + pos / V, k = pos % V;
+                if (j < nmine && ((vcm_p >> k) & 1u)) {
+                    const int c = lane * V + k;
+                    const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
+                    if (at < (uint32_t)kCap)
+                        cp_async4(list_s + (at * TC + c) * 4u, row_ptr(lb_p, j) + k);
+                }
             }
         }
+        cp_async_commit();
     };
 
     // rank the pending tile's listed bins: one thread per coordinate
@@ -297,20 +318,22 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
         const bool lvn = tn < ntiles && tn * TC + lane * V < d;
         const char *lbn = lvn ? lane_base(tn) : lb;
 
-        // One pass over this warp's rows, batch by batch: fn(x, j, u) for
-        // every row; each register is refilled right after it is used.
-        auto sweep = [&](auto fn) {
+        // One pass over this warp's rows, batch by batch: pre(j0) at the start
+        // of a batch, fn(x, j, u) for every row; each register is refilled
+        // right after it is used.
+        auto sweep = [&](auto pre, auto fn) {
             auto batch = [&](auto lastc, int j0) {
                 constexpr bool LAST = decltype(lastc)::value;
+                pre(j0);
 #pragma unroll
                 for (int u = 0; u < kU; ++u) {
                     if constexpr (LAST) {
                         if (j0 + u < nmine) fn(xa[u], j0 + u, u);
-                        xa[u] = (lvn && u < nmine) ? load_row<V>(row_ptr(lbn, u)) : T{};
+                        if (lvn && u < nmine) xa[u] = load_row<V>(row_ptr(lbn, u));
                     } else {
                         fn(xa[u], j0 + u, u);
                         const int jn = j0 + kU + u;
-                        xa[u] = (lv && jn < nmine) ? load_row<V>(row_ptr(lb, jn)) : T{};
+                        if (lv && jn < nmine) xa[u] = load_row<V>(row_ptr(lb, jn));
                     }
                 }
             };
@@ -324,7 +347,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             float sm[V], se[V];
 #pragma unroll
             for (int k = 0; k < V; ++k) sm[k] = se[k] = 0.f;
-            sweep([&](const T &x, int, int) {
+            sweep([](int) {}, [&](const T &x, int, int) {
 #pragma unroll
                 for (int k = 0; k < V; ++k) {
                     float ns, ne;
@@ -400,11 +423,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             // ---- sweep: the pending tile's members (old tag words), then
             // VH for this tile (histogram, new tag words, NaN check)
             uint32_t nanf = 0u, tacc = 0u;
-            sweep([&](const T &x, int j, int u) {
-                if (u % RPW == 0) {
-                    const uint32_t z = tag_match(tags[((j / RPW) * kWarps + w) * 32 + lane], vbx_p);
-                    if (z) capture(z, j / RPW);
-                }
+            sweep([](int) {}, [&](const T &x, int j, int u) {
                 uint32_t bb[V];
 #pragma unroll
                 for (int k = 0; k < V; ++k) {
@@ -436,7 +455,6 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     if ((u & 3) == 3 || j + 1 >= nmine) tags[((j >> 2) * kWarps + w) * 32 + lane] = tacc;
                 }
             });
-            cp_async_commit();
             if (nanf) {
 #pragma unroll
                 for (int k = 0; k < V; ++k) atomicOr(&S(S_NAN, lane * V + k), 1u);
@@ -457,15 +475,16 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             __syncthreads();                                        // (R)
             for (int c = tid; c < TC; c += kThreads) S(S_LCNT, c) = 0u;
 
-            // ---- B1: per-warp partial sums over bins [16w, 16w + 16)
+            // ---- B1: per-warp partial sums over bins [kBPW*w, kBPW*w + kBPW)
             {
                 uint32_t ps[NP];
 #pragma unroll
                 for (int p = 0; p < NP; ++p) ps[p] = 0u;
 #pragma unroll
-                for (int b = 0; b < 16; ++b)
+                for (int b = 0; b < kBPW; ++b)
+                    if (w * kBPW + b < kNB)
 #pragma unroll
-                    for (int p = 0; p < NP; ++p) ps[p] += hist[((w * 16 + b) * NP + p) * 32 + lane];
+                        for (int p = 0; p < NP; ++p) ps[p] += hist[((w * kBPW + b) * NP + p) * 32 + lane];
 #pragma unroll
                 for (int k = 0; k < V; ++k)
                     list[w * TC + lane * V + k] = (ps[k / 2] >> (16 * (k & 1))) & 0xFFFFu;
@@ -488,10 +507,10 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     const int lc = c / V, k = c % V;
                     const uint32_t *h = hist + (k / 2) * 32 + lc;
                     const int shf = 16 * (k & 1);
-                    int bin = owner * 16 + 15;
+                    int bin = min(owner * kBPW + kBPW, kNB) - 1;
                     uint32_t cnt = 0u;
                     bool f2 = false;
-                    for (int b = owner * 16; b < owner * 16 + 16; ++b) {
+                    for (int b = owner * kBPW; b < min(owner * kBPW + kBPW, kNB); ++b) {
                         const uint32_t cb = (h[b * NP * 32] >> shf) & 0xFFFFu;
                         const bool hit = !f2 && rem < cb;
                         if (hit) {
@@ -532,6 +551,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             c0_p = c0;
             vbx_p = vbx;
             vcm_p = vcm;
+            capture_members();
 
             if (__syncthreads_or(need_general)) {
                 // ---- exact fallback passes (rare), values re-read from global memory
@@ -654,13 +674,8 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
         }
     }
     if constexpr (MODE == 0) {
-        // the last tile's members: scan its tags, then rank
+        // the last tile's listed members are ranked once their copies land
         if (have_p) {
-            for (int q = 0; q < nwords; ++q) {
-                const uint32_t z = tag_match(tags[(q * kWarps + w) * 32 + lane], vbx_p);
-                if (z) capture(z, q);
-            }
-            cp_async_commit();
             cp_async_wait_all();
             __syncthreads();
             rank_pending();
