@@ -13,24 +13,27 @@
 // batch's row as soon as it is read, and the last batch of a tile refills
 // with the first rows of the CTA's next tile, whose loads then overlap this
 // tile's remaining phases.  Shared memory holds one tag byte per value, the
-// histograms and small per-coordinate state; two CTAs share an SM.
+// histograms, the member lists and small per-coordinate state; two CTAs of
+// 12 warps share an SM.
 //
 // Lower median, exact (IEEE totalOrder through a monotone uint32 key; the key
 // map is a bijection, so the output has the chosen element's bits).  Per
 // tile:
-//   S   sample: key range of the first two rows of every warp (16 values per
+//   S   sample: key range of the first two rows of every warp (24 values per
 //       coordinate).
 //   VH  value-space histogram of every value: bins 1..125 evenly over the
 //       sample range, 0 and 126 catch everything below / above (vbin_bits);
 //       each value's bin is kept as a tag byte; NaNs are detected.  Counters
 //       are the 16-bit halves of words in per-lane columns, so the 32 shared
 //       atomics of a warp instruction hit 32 different banks.
-//   B   bin search: per-warp partial sums over 16 bins, then one thread per
+//   B   bin search: per-warp partial sums over kBPW bins, then one thread per
 //       coordinate finds the bin that holds the target rank, the rank inside
 //       it and its count.
-//   VC  four tag bytes are compared per word; the bin's members (about n/100)
-//       are re-read from global memory (L2) into a list of at most kCap keys
-//       per coordinate, which 8 threads per coordinate rank directly.
+//   VC  right after the bin search, four tag bytes are compared per word; the
+//       bin's members (about n/80) are copied from global memory (the tile is
+//       still in L2) into a list of at most kCap values per coordinate by
+//       4-byte cp.async; they land during the next tile's sweep, after which
+//       one thread per coordinate sorts its keys in registers.
 // Exact fallback for the coordinates that need it (NaN seen, degenerate or
 // non-finite sample range, more than kCap members in the bin), values
 // re-read from global memory:
