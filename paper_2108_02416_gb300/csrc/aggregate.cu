@@ -9,10 +9,10 @@
 // segments of 455 rows that lie 45 MB apart runs at about 4.9 TB/s on GB300,
 // 512-byte segments at 7.0; staging whole tiles in shared memory would limit
 // the segments to 128 bytes.)  Each value is used once, from registers: rows
-// come in batches of kU per thread, every register refilled with the next
-// batch's row as soon as it is read, and the last batch of a tile refills
-// with the first rows of the CTA's next tile, whose loads then overlap this
-// tile's remaining phases.  Shared memory holds one tag byte per value, the
+// come in batches of kU (8, or 24 for V <= 2 with one CTA per SM) per thread, every
+// register refilled with the next batch's row as soon as it is read, and the
+// last batch of a tile refills with the first rows of the CTA's next tile,
+// whose loads then overlap this tile's remaining phases.  Shared memory holds one tag byte per value, the
 // histograms, the member lists and small per-coordinate state; two CTAs of
 // 12 warps share an SM.
 //
@@ -31,17 +31,17 @@
 //       it and its count.
 //   VC  right after the bin search, four tag bytes are compared per word; the
 //       bin's members (about n/80) are copied from global memory (the tile is
-//       still in L2) into a list of at most kCap values per coordinate by
+//       still in L2) into a list of at most CAP values per coordinate (4096 / TC) by
 //       4-byte cp.async; they land during the next tile's sweep, after which
 //       one thread per coordinate sorts its keys in registers.
 // Exact fallback for the coordinates that need it (NaN seen, degenerate or
-// non-finite sample range, more than kCap members in the bin), values
+// non-finite sample range, more than CAP members in the bin), values
 // re-read from global memory:
 //   VM  exact key range [lo, hi] of the crowded bin's members
 //   KA  key range [lo, hi] of all values
 //   KH  128 equal-width key-space bins over [lo, hi]; the bin holding the
 //       rank becomes [lo, hi] (each pass shrinks the range by 2^7)
-//   KC  the at most kCap keys left in [lo, hi] are listed and ranked.
+//   KC  the at most CAP keys left in [lo, hi] are listed and ranked.
 // The fallback loop is bounded (kMaxPasses); every wait is a block barrier.
 #include <type_traits>
 
@@ -54,8 +54,8 @@ namespace {
 constexpr int kThreads = 384;
 constexpr int kWarps = kThreads / 32;     // row slots of a CTA
 constexpr int kBPW = (kNB + kWarps - 1) / kWarps;   // histogram bins per warp in the bin search
-constexpr int kU = 8;                     // rows per load batch and thread
 constexpr int kMaxPasses = 12;            // fallback: VM/KA, at most 5 KH, KC
+constexpr int kListWords = 4096;          // member lists: 32, 64 or 128 per coordinate
 
 // per-coordinate state, arrays of TC words
 enum { S_MIN, S_MAX, S_NAN, S_LCNT, S_MODE, S_BIN, S_REM, S_CNT, S_LO, S_HI, S_PCNT, S_PREM,
@@ -139,6 +139,7 @@ struct Geo {
     static constexpr int NP = V >= 2 ? V / 2 : 1;     // histogram words per (bin, lane)
     static constexpr int SHB = NP == 2 ? 8 : 7;       // log2 of the bytes per histogram row
     static constexpr int RPW = 4 / V;                 // rows per tag word
+    static constexpr int CAP = kListWords / TC;       // list entries per coordinate
 };
 
 struct Layout {
@@ -155,7 +156,7 @@ __host__ __device__ inline Layout make_layout(int64_t f)
     size_t o = 0;
     L.tags = o; o += (size_t)jw * kWarps * 32 * 4;
     L.hist = o; o += (size_t)kNB * G::NP * 32 * 4;
-    L.list = o; o += (size_t)kCap * G::TC * 4;       // also the bin-search and mean partials
+    L.list = o; o += (size_t)kListWords * 4;         // also the bin-search and mean partials
     L.state = o; o += (size_t)kStateWords * G::TC * 4;
     L.rows = o; o += ((size_t)f * 2 + 15) / 16 * 16;
     L.total = o;
@@ -169,12 +170,15 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
 {
     using G = Geo<V>;
     using T = typename Vec<V>::T;
-    constexpr int TC = G::TC, NP = G::NP, SHB = G::SHB, RPW = G::RPW;
+    constexpr int TC = G::TC, NP = G::NP, SHB = G::SHB, RPW = G::RPW, CAP = G::CAP;
+    // rows per load batch and thread: deeper when one CTA has the SM's
+    // registers and rows are narrow
+    constexpr int kU = (MINB >= 2 || V == 4) ? 8 : 24;
     extern __shared__ __align__(16) unsigned char smem[];
     const Layout L = make_layout<V>(f);
     uint32_t *tags = reinterpret_cast<uint32_t *>(smem + L.tags);     // [word][kWarps][32]
     uint32_t *hist = reinterpret_cast<uint32_t *>(smem + L.hist);     // [kNB][NP][32]
-    uint32_t *list = reinterpret_cast<uint32_t *>(smem + L.list);     // [kCap][TC]
+    uint32_t *list = reinterpret_cast<uint32_t *>(smem + L.list);     // [CAP][TC]
     uint32_t *st = reinterpret_cast<uint32_t *>(smem + L.state);      // [kStateWords][TC]
     uint16_t *rows = reinterpret_cast<uint16_t *>(smem + L.rows);
     __shared__ int warp_tot[kWarps];
@@ -274,7 +278,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 if (j < nmine && ((vcm_p >> k) & 1u)) {
                     const int c = lane * V + k;
                     const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
-                    if (at < (uint32_t)kCap)
+                    if (at < (uint32_t)CAP)
                         cp_async4(list_s + (at * TC + c) * 4u, row_ptr(lb_p, j) + k);
                 }
             }
@@ -282,34 +286,38 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
         cp_async_commit();
     };
 
-    // rank the pending tile's listed bins: one thread per coordinate
+    // Rank the pending tile's listed bins.  Lists of at most 16 keys (the
+    // common case): one thread per coordinate sorts them in registers.
+    // Longer lists: kThreads/TC threads per coordinate, each counting, for its
+    // candidates, the listed keys below and at them.
     auto rank_pending = [&]() {
         for (int c = tid; c < TC; c += kThreads) {
             const uint32_t cnt = S(S_PCNT, c);
-            if (cnt == 0u) continue;
+            if (cnt == 0u || cnt > 16u) continue;
             const uint32_t rk = S(S_PREM, c);
-            uint32_t res = 0u;
-            if (cnt <= 16u) {
-                uint32_t y[16];
+            uint32_t y[16];
 #pragma unroll
-                for (int e = 0; e < 16; ++e) y[e] = (uint32_t)e < cnt ? to_key(list[e * TC + c]) : 0xffffffffu;
-                sort16(y);
-                res = y[0];
+            for (int e = 0; e < 16; ++e) y[e] = (uint32_t)e < cnt ? to_key(list[e * TC + c]) : 0xffffffffu;
+            sort16(y);
+            uint32_t res = y[0];
 #pragma unroll
-                for (int e = 1; e < 16; ++e) res = (uint32_t)e == rk ? y[e] : res;
-            } else {
-                for (uint32_t e = 0; e < cnt; ++e) {
-                    const uint32_t x = to_key(list[e * TC + c]);
-                    uint32_t lt = 0u, le = 0u;
-                    for (uint32_t t2 = 0; t2 < cnt; ++t2) {
-                        const uint32_t y = to_key(list[t2 * TC + c]);
-                        lt += y < x;
-                        le += y <= x;
-                    }
-                    if (lt <= rk && rk < le) res = x;
-                }
-            }
+            for (int e = 1; e < 16; ++e) res = (uint32_t)e == rk ? y[e] : res;
             out[c0_p + c] = __uint_as_float(from_key(res));
+        }
+        constexpr int P = kThreads / TC;
+        const int c = tid % TC, e0 = tid / TC;
+        const uint32_t cnt = e0 < P ? S(S_PCNT, c) : 0u;
+        if (cnt <= 16u) return;
+        const uint32_t rk = S(S_PREM, c);
+        for (uint32_t e = (uint32_t)e0; e < cnt; e += P) {
+            const uint32_t x = to_key(list[e * TC + c]);
+            uint32_t lt = 0u, le = 0u;
+            for (uint32_t t2 = 0; t2 < cnt; ++t2) {
+                const uint32_t y = to_key(list[t2 * TC + c]);
+                lt += y < x;
+                le += y <= x;
+            }
+            if (lt <= rk && rk < le) out[c0_p + c] = __uint_as_float(from_key(x));
         }
     };
 
@@ -527,7 +535,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     S(S_REM, c) = rem;
                     S(S_CNT, c) = cnt;
                     S(S_PREM, c) = rem;
-                    const bool vcm = cnt <= (uint32_t)kCap;
+                    const bool vcm = cnt <= (uint32_t)CAP;
                     S(S_MODE, c) = vcm ? M_VC : M_VM;
                     pc = vcm ? cnt : 0u;
                 }
@@ -575,22 +583,31 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                             const uint32_t vb = S(S_BIN, c);
                             const uint8_t *tb = reinterpret_cast<const uint8_t *>(tags);
                             uint32_t a = 0xffffffffu, bmax = 0u;
-                            for (int j = 0; j < nmine; ++j) {
-                                if (md == M_VM) {
-                                    const int q = j / RPW, p = (j % RPW) * V + k;
-                                    if (tb[((q * kWarps + w) * 32 + lane) * 4 + p] != vb) continue;
-                                }
-                                const uint32_t key = to_key(reread(j, k));
-                                if (md == M_VM || md == M_KA) {
-                                    a = min(a, key);
-                                    bmax = max(bmax, key);
-                                } else if (key - lo <= W) {
-                                    if (md == M_KH) {
-                                        atomicAdd(hist + (((key - lo) >> sh) * NP + k / 2) * 32 + lane,
-                                                  (k & 1) ? 0x10000u : 1u);
-                                    } else {
-                                        const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
-                                        if (at < (uint32_t)kCap) list[at * TC + c] = key;
+                            for (int j0 = 0; j0 < nmine; j0 += 8) {
+                                uint32_t vals[8];
+#pragma unroll
+                                for (int u = 0; u < 8; ++u)        // eight loads in flight
+                                    if (j0 + u < nmine) vals[u] = reread(j0 + u, k);
+#pragma unroll
+                                for (int u = 0; u < 8; ++u) {
+                                    const int j = j0 + u;
+                                    if (j >= nmine) break;
+                                    if (md == M_VM) {
+                                        const int q = j / RPW, p = (j % RPW) * V + k;
+                                        if (tb[((q * kWarps + w) * 32 + lane) * 4 + p] != vb) continue;
+                                    }
+                                    const uint32_t key = to_key(vals[u]);
+                                    if (md == M_VM || md == M_KA) {
+                                        a = min(a, key);
+                                        bmax = max(bmax, key);
+                                    } else if (key - lo <= W) {
+                                        if (md == M_KH) {
+                                            atomicAdd(hist + (((key - lo) >> sh) * NP + k / 2) * 32 + lane,
+                                                      (k & 1) ? 0x10000u : 1u);
+                                        } else {
+                                            const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
+                                            if (at < (uint32_t)CAP) list[at * TC + c] = key;
+                                        }
                                     }
                                 }
                             }
@@ -615,7 +632,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                                 rk = krank;
                                 cnt = (uint32_t)n;
                             }
-                            nm = lo == hi ? M_DONE : (cnt <= (uint32_t)kCap ? M_KC : M_KH);
+                            nm = lo == hi ? M_DONE : (cnt <= (uint32_t)CAP ? M_KC : M_KH);
                         } else if (md == M_KH) {
                             const uint32_t W = hi - lo;
                             const int bits = 32 - __clz(W);
@@ -634,9 +651,9 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                             const uint64_t top = (uint64_t)nlo + ((1ull << sh) - 1ull);
                             hi = top < (uint64_t)hi ? (uint32_t)top : hi;
                             lo = nlo;
-                            nm = lo == hi ? M_DONE : (cnt <= (uint32_t)kCap ? M_KC : M_KH);
+                            nm = lo == hi ? M_DONE : (cnt <= (uint32_t)CAP ? M_KC : M_KH);
                         } else if (md == M_KC) {
-                            const uint32_t m = min(cnt, (uint32_t)kCap);
+                            const uint32_t m = min(cnt, (uint32_t)CAP);
                             for (uint32_t e = 0; e < m; ++e) {
                                 const uint32_t x = list[e * TC + c];
                                 uint32_t lt = 0u, le = 0u;

@@ -31,6 +31,55 @@ using namespace aspis;
 
 namespace {
 
+// Host-to-device copies of the round's inputs are split over kLanes streams
+// so that several copy engines move them at once; the caller's stream waits
+// for all of them.  Streams and events are created once per device.
+constexpr int kLanes = 4;
+struct CopyLanes {
+    bool ready = false;
+    cudaStream_t s[kLanes];
+    cudaEvent_t start, done[kLanes];
+};
+std::mutex g_lanes_mu;
+CopyLanes g_lanes[64];
+
+cudaError_t h2d_split(void *dst, const void *src, size_t bytes, cudaStream_t st)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64 || bytes < ((size_t)64 << 20))
+        return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, st);
+    std::lock_guard<std::mutex> g(g_lanes_mu);
+    CopyLanes &L = g_lanes[dev];
+    if (!L.ready) {
+        for (int i = 0; i < kLanes; ++i) {
+            if ((e = cudaStreamCreateWithFlags(&L.s[i], cudaStreamNonBlocking)) != cudaSuccess) return e;
+            if ((e = cudaEventCreateWithFlags(&L.done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
+        }
+        if ((e = cudaEventCreateWithFlags(&L.start, cudaEventDisableTiming)) != cudaSuccess) return e;
+        L.ready = true;
+    }
+    if ((e = cudaEventRecord(L.start, st)) != cudaSuccess) return e;
+    const size_t chunk = (bytes / kLanes + 4095) / 4096 * 4096;
+    for (int i = 0; i < kLanes; ++i) {
+        const size_t off = (size_t)i * chunk;
+        if (off >= bytes) break;
+        const size_t len = bytes - off < chunk ? bytes - off : chunk;
+        if ((e = cudaStreamWaitEvent(L.s[i], L.start, 0)) != cudaSuccess) return e;
+        e = cudaMemcpyAsync(static_cast<char *>(dst) + off, static_cast<const char *>(src) + off, len,
+                            cudaMemcpyHostToDevice, L.s[i]);
+        if (e != cudaSuccess) return e;
+        if ((e = cudaEventRecord(L.done[i], L.s[i])) != cudaSuccess) return e;
+        if ((e = cudaStreamWaitEvent(st, L.done[i], 0)) != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
+}  // namespace
+
+namespace {
+
 inline aspis_status cuda_status(cudaError_t e) { return e == cudaSuccess ? ASPIS_OK : ASPIS_E_CUDA; }
 
 aspis_status check_assignment(const aspis_assignment *a)
@@ -166,8 +215,7 @@ extern "C" aspis_status aspis_round_host(const float *host_copies, float *dev_co
     if ((s = check_copies(dev_copies, d, ld, a)) != ASPIS_OK) return s;
     cudaStream_t st = (cudaStream_t)stream;
     const size_t bytes = sizeof(float) * (size_t)(a->f * a->r) * (size_t)ld;
-    if (cudaMemcpyAsync(dev_copies, host_copies, bytes, cudaMemcpyHostToDevice, st) != cudaSuccess)
-        return ASPIS_E_CUDA;
+    if (h2d_split(dev_copies, host_copies, bytes, st) != cudaSuccess) return ASPIS_E_CUDA;
     s = aspis_round(dev_copies, d, ld, a, file_neq, adj, det, sel, mode, dev_out, stream);
     if (s != ASPIS_OK) return s;
     if (cudaMemcpyAsync(host_out, dev_out, sizeof(float) * (size_t)d, cudaMemcpyDeviceToHost,
