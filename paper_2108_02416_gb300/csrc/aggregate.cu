@@ -51,9 +51,6 @@
 namespace aspis {
 namespace {
 
-constexpr int kThreads = 384;
-constexpr int kWarps = kThreads / 32;     // row slots of a CTA
-constexpr int kBPW = (kNB + kWarps - 1) / kWarps;   // histogram bins per warp in the bin search
 constexpr int kMaxPasses = 12;            // fallback: VM/KA, at most 5 KH, KC
 constexpr int kListWords = 4096;          // member lists: 32, 64 or 128 per coordinate
 
@@ -146,10 +143,11 @@ struct Layout {
     size_t tags, hist, list, state, rows, total;
 };
 
-template <int V>
+template <int V, int NT>
 __host__ __device__ inline Layout make_layout(int64_t f)
 {
     using G = Geo<V>;
+    constexpr int kWarps = NT / 32;
     Layout L{};
     const int64_t per_slot = (f + kWarps - 1) / kWarps;
     const int64_t jw = (per_slot + G::RPW - 1) / G::RPW;     // tag words per thread
@@ -163,19 +161,21 @@ __host__ __device__ inline Layout make_layout(int64_t f)
     return L;
 }
 
-template <int V, int MINB, bool W32, int MODE>
-__global__ void __launch_bounds__(kThreads, MINB)
+template <int V, int MINB, bool W32, int MODE, int NT>
+__global__ void __launch_bounds__(NT, MINB)
 aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, int64_t ld,
                  const int8_t *__restrict__ sel, aspis_detection *det, float *__restrict__ out)
 {
     using G = Geo<V>;
     using T = typename Vec<V>::T;
     constexpr int TC = G::TC, NP = G::NP, SHB = G::SHB, RPW = G::RPW, CAP = G::CAP;
-    // rows per load batch and thread: deeper when one CTA has the SM's
-    // registers and rows are narrow
+    constexpr int kThreads = NT, kWarps = NT / 32;           // warps = row slots of a CTA
+    constexpr int kBPW = (kNB + kWarps - 1) / kWarps;        // bins per warp in the bin search
+    // rows per load batch and thread: deeper for narrow rows when one CTA
+    // has the SM's registers
     constexpr int kU = (MINB >= 2 || V == 4) ? 8 : 24;
     extern __shared__ __align__(16) unsigned char smem[];
-    const Layout L = make_layout<V>(f);
+    const Layout L = make_layout<V, NT>(f);
     uint32_t *tags = reinterpret_cast<uint32_t *>(smem + L.tags);     // [word][kWarps][32]
     uint32_t *hist = reinterpret_cast<uint32_t *>(smem + L.hist);     // [kNB][NP][32]
     uint32_t *list = reinterpret_cast<uint32_t *>(smem + L.list);     // [CAP][TC]
@@ -711,26 +711,26 @@ size_t smem_cap()
     return (size_t)cap - 1024;        // static shared memory and reserve
 }
 
-template <int V, int MINB, bool W32, int MODE>
+template <int V, int MINB, bool W32, int MODE, int NT>
 cudaError_t try_launch(bool &launched, const float *copies, int64_t f, int r, int64_t d,
                        int64_t ld, const int8_t *sel, aspis_detection *det, float *out,
                        cudaStream_t stream)
 {
     launched = false;
-    const Layout L = make_layout<V>(f);
+    const Layout L = make_layout<V, NT>(f);
     if (L.total > smem_cap()) return cudaSuccess;
-    auto kern = aggregate_kernel<V, MINB, W32, MODE>;
+    auto kern = aggregate_kernel<V, MINB, W32, MODE, NT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)L.total);
     if (e != cudaSuccess) return e;
     int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, L.total);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, NT, L.total);
     if (e != cudaSuccess) return e;
     if (per_sm < MINB) return cudaSuccess;        // the next configuration is tried
     const int64_t ntiles = (d + Geo<V>::TC - 1) / Geo<V>::TC;
     int64_t grid = (int64_t)sm_count() * per_sm;
     if (grid > ntiles) grid = ntiles;
-    kern<<<(unsigned)grid, kThreads, L.total, stream>>>(copies, f, r, d, ld, sel, det, out);
+    kern<<<(unsigned)grid, NT, L.total, stream>>>(copies, f, r, d, ld, sel, det, out);
     launched = true;
     return cudaGetLastError();
 }
@@ -741,23 +741,23 @@ cudaError_t launch_mode(int align, const float *copies, int64_t f, int r, int64_
 {
     bool ok = false;
     cudaError_t e = cudaSuccess;
-#define ASPIS_TRY(V, MB)                                                                        \
-    e = try_launch<V, MB, W32, MODE>(ok, copies, f, r, d, ld, sel, det, out, stream);           \
+#define ASPIS_TRY(V, MB, NT)                                                                    \
+    e = try_launch<V, MB, W32, MODE, NT>(ok, copies, f, r, d, ld, sel, det, out, stream);       \
     if (e != cudaSuccess || ok) return e;
     if (align >= 4) {
-        ASPIS_TRY(4, 2)
+        ASPIS_TRY(4, 2, 384)
     }
     if (align >= 2) {
-        ASPIS_TRY(2, 2)
+        ASPIS_TRY(2, 2, 384)
     }
     if (align >= 4) {
-        ASPIS_TRY(4, 1)
+        ASPIS_TRY(4, 1, 384)
     }
     if (align >= 2) {
-        ASPIS_TRY(2, 1)
+        ASPIS_TRY(2, 1, 384)
     }
-    ASPIS_TRY(1, 2)
-    ASPIS_TRY(1, 1)
+    ASPIS_TRY(1, 2, 384)
+    ASPIS_TRY(1, 1, 384)
 #undef ASPIS_TRY
     return cudaErrorInvalidValue;
 }
