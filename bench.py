@@ -15,6 +15,10 @@ between rounds.
 
 Prints one JSON line (rank 0).  With N > 1 (torchrun) every rank runs an
 independent replica on its own GPU; there is no data-path collective.
+
+Besides the step, the line reports the model update that follows it
+(aspis_sgd: Eq. 1 with momentum 0.9 on the round's output), timed alone with
+L2 flushed before every launch (key "update"); it is not part of the step.
 """
 from __future__ import annotations
 
@@ -51,6 +55,8 @@ def parse():
     p.add_argument("--e2e-steps", type=int, default=5)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
+    p.add_argument("--no-update", action="store_true",
+                   help="skip the separate timing of the model update")
     p.add_argument("--cpu-seconds", type=float, default=12.0,
                    help="target CPU time of the oracle baseline sample")
     return p.parse_args()
@@ -311,6 +317,37 @@ def main():
     agg_traffic = profile_traffic("aggregate_kernel", w.name, n_sel * w.d,
                                   os.path.join(csrc, "aggregate.cu"))
 
+    # ---- the model update on the round's output, timed alone: w, v <- Eq. 1
+    # with momentum 0.9; 20 bytes per coordinate (read g, w, v; write w, v)
+    update = None
+    if not args.no_update:
+        wp = torch.zeros(w.d, dtype=torch.float32, device=dev)
+        vp = torch.zeros(w.d, dtype=torch.float32, device=dev)
+        fl = flush if flush is not None else torch.empty(256 * 1024 * 1024, dtype=torch.uint8,
+                                                         device=dev)
+        uev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+        stream.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(stream):
+            for _ in range(max(3, args.warmup)):
+                ap.aspis_sgd(buf.out, wp, vp, 0.01, 0.9, stream)
+            for k in range(args.steps):
+                fl.zero_()
+                uev[k][0].record(stream)
+                ap.aspis_sgd(buf.out, wp, vp, 0.01, 0.9, stream)
+                uev[k][1].record(stream)
+        torch.cuda.synchronize()
+        upd_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in uev)
+        upd_bytes = 20 * w.d
+        upd_gbs = upd_bytes / (upd_ms * 1e-3) / 1e9
+        update = {"kernel": "sgd_vec_kernel (aspis_sgd, momentum 0.9)", "bound": "hbm",
+                  "ms": upd_ms, "achieved": upd_gbs, "peak": peak, "unit": "GB/s",
+                  "frac": upd_gbs / peak, "peak_kind": peak_kind,
+                  "algorithmic_bytes": upd_bytes, "launches": args.steps,
+                  "l2": "flushed before every launch"}
+        if flush is None:
+            del fl
+        del wp, vp
+
     # ---- end to end through aspis_round_host from pinned host memory
     e2e = None
     if not args.no_e2e:
@@ -385,6 +422,7 @@ def main():
         "gpu_launches": launches_per_round * args.steps,
         "e2e": e2e,
         "cpu_baseline": cpu,
+        "update": update,
     }
     json_line(line)
     if dist:

@@ -235,6 +235,30 @@ aspis_status aspis_round_host(const float *host_copies, float *dev_copies,
                               float *dev_out, float *host_out,
                               aspis_detection *host_det, void *stream);
 
+/* The model update that follows the aggregation (Section 2, Eq. 1, with
+ * the aggregate of Algorithm 1 in place of the batch gradient), with the
+ * heavy-ball momentum of the experiments (Appendix B: momentum 0.9).  For
+ * every coordinate c < d:
+ *     mu != 0:  v[c] <- RN(mu * v[c] + g[c]);  w[c] <- RN(w[c] - eta * v[c])
+ *     mu == 0:  w[c] <- RN(w[c] - eta * g[c])   (Eq. 1; v is not touched)
+ * where RN rounds the exact value once to fp32 (round to nearest even), so
+ * results are bitwise reproducible; NaN and infinity follow IEEE-754.
+ *   g    device [d] fp32, in: the aggregated gradient (aspis_aggregate's out)
+ *   w    device [d] fp32, in/out: the parameters
+ *   v    device [d] fp32, in/out: the momentum buffer (zeros before the first
+ *        update); may be NULL when mu == 0
+ *   eta  the step eta_t of this iteration (the experiments' schedules are
+ *        x * y^floor(t/z), computed by the caller)
+ * g, w and v are each either the same array or disjoint; a partial overlap,
+ * d < 0 or a missing pointer returns ASPIS_E_INVAL, d == 0 does nothing.
+ * 16-byte aligned pointers take the 128-bit path (any d; the last d % 4
+ * coordinates one by one), others a 4-byte path.  Reads 12 bytes per
+ * coordinate and writes 8 (8 and 4 when mu == 0).  No counterpart of a
+ * separate call in the paper, whose PS applies this update right after the
+ * aggregation. */
+aspis_status aspis_sgd(const float *g, float *w, float *v, int64_t d, float eta,
+                       float mu, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -16,6 +16,7 @@ Detection for Distributed Learning"):
 * :func:`max_cliques_brute` / :func:`max_cliques_bk` -- Algorithm 3
 * :func:`select`            -- Algorithm 1, Case 1 / Case 2 (Eq. 2)
 * :func:`aggregate`, :func:`lower_median`, :func:`mean` -- Algorithm 1 updates
+* :func:`sgd`               -- the model update with the aggregate (Eq. 1, momentum)
 * :func:`run_round`         -- the whole step in the paper's order
 """
 from __future__ import annotations
@@ -45,7 +46,7 @@ def build_oracle(force: bool = False) -> str:
         return _LIB_PATH
     tmp = _LIB_PATH + f".tmp{os.getpid()}"
     subprocess.check_call(["gcc", "-O2", "-std=c11", "-shared", "-fPIC", "-pthread",
-                           _SRC, "-o", tmp])
+                           _SRC, "-o", tmp, "-lm"])
     os.replace(tmp, _LIB_PATH)
     return _LIB_PATH
 
@@ -70,6 +71,7 @@ def _load():
             lib.oracle_aggregate.argtypes = [P, i64, i32, i64, P, i32, i64, i64, P, i32]
             lib.oracle_lower_median.argtypes = [P, i64, i64, P]
             lib.oracle_mean.argtypes = [P, i64, i64, P]
+            lib.oracle_sgd.argtypes = [P, P, P, i64, ctypes.c_float, ctypes.c_float]
             _lib = lib
     return _lib
 
@@ -218,6 +220,24 @@ def mean(vals: np.ndarray) -> np.ndarray:
     if rc != OK:
         raise ValueError(f"oracle_mean failed: {rc}")
     return out[:m]
+
+
+def sgd(g: np.ndarray, w: np.ndarray, v: np.ndarray | None, eta: float, mu: float):
+    """One update w, v <- (Eq. 1 with momentum) on copies; returns (w', v').
+
+    eta and mu are rounded to fp32 first, as the library receives them.
+    With mu == 0, v is returned unchanged (None stays None)."""
+    g = np.ascontiguousarray(g, dtype=np.float32)
+    w2 = np.array(w, dtype=np.float32, copy=True)
+    v2 = None if v is None else np.array(v, dtype=np.float32, copy=True)
+    m = g.size
+    if w2.size != m or (v2 is not None and v2.size != m):
+        raise ValueError("g, w and v must have the same length")
+    rc = _load().oracle_sgd(_ptr(g), _ptr(w2), None if v2 is None else _ptr(v2), m,
+                            float(np.float32(eta)), float(np.float32(mu)))
+    if rc != OK:
+        raise ValueError(f"oracle_sgd failed: {rc}")
+    return w2, v2
 
 
 @dataclass

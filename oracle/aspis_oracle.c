@@ -20,6 +20,8 @@
  *   oracle_select              Algorithm 1: Case 1 honest copy / Case 2 majority (Eq. 2)
  *   oracle_lower_median        coordinate-wise median of the chosen gradients (Algorithm 1, Case 2)
  *   oracle_mean                average of the chosen gradients (Algorithm 1, Case 1)
+ *   oracle_sgd                 the model update with the aggregate (Section 2, Eq. 1;
+ *                              Algorithm 1), with heavy-ball momentum (Appendix B)
  *
  * Readings where the paper is silent (each also listed in the design notes):
  *   - file i <-> the i-th r-subset of workers in lexicographic order; Example 1
@@ -34,6 +36,10 @@
  *     the selected element.
  *   - Case 1 chooses the honest copy with the lowest slot; files with no
  *     honest worker are dropped.
+ *   - the momentum of the experiments (0.9) is heavy-ball momentum without
+ *     dampening, v <- mu*v + g, w <- w - eta*v, as in the paper's PyTorch
+ *     framework; each of the two results is the exact value rounded once
+ *     to fp32.
  *
  * Parity status: every function here is pinned by tests (closed-form counts,
  * Example 1, the Figure 3 graphs, Theorem 1, brute force, NetworkX clique
@@ -41,6 +47,7 @@
  * facts: the plurality rule when no strict majority exists and the rounding
  * of the mean (checked against an exactly-rounded sum within a tolerance).
  */
+#include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
@@ -465,6 +472,30 @@ int oracle_mean(const float *vals, int64_t n, int64_t m, float *out)
         double acc = 0.0;
         for (int64_t i = 0; i < n; ++i) acc += (double)vals[i * m + c];
         out[c] = (float)(acc / (double)n);
+    }
+    return ORACLE_OK;
+}
+
+/* One model update with the aggregated gradient g, over m coordinates.
+ * Eq. 1 (Section 2) moves w against the batch gradient with step eta; the
+ * PS of Algorithm 1 uses the aggregate of the chosen copies in its place.
+ * The experiments add momentum 0.9 (Appendix B), read as heavy-ball
+ * momentum:
+ *     v[c] <- mu * v[c] + g[c]        then        w[c] <- w[c] - eta * v[c],
+ * each the exact real value rounded once to fp32 (C99 fmaf is exactly
+ * that).  mu == 0 is Eq. 1 itself, w[c] <- w[c] - eta * g[c], and v is not
+ * touched (it may be NULL). */
+int oracle_sgd(const float *g, float *w, float *v, int64_t m, float eta, float mu)
+{
+    if (m < 0 || (m > 0 && (!g || !w))) return ORACLE_EINVAL;
+    if (mu != 0.0f && m > 0 && !v) return ORACLE_EINVAL;
+    for (int64_t c = 0; c < m; ++c) {
+        if (mu != 0.0f) {
+            v[c] = fmaf(mu, v[c], g[c]);
+            w[c] = fmaf(-eta, v[c], w[c]);
+        } else {
+            w[c] = fmaf(-eta, g[c], w[c]);
+        }
     }
     return ORACLE_OK;
 }

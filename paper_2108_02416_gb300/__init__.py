@@ -16,6 +16,7 @@ The call names mirror the C entry points:
   aspis_round(...)                          the four device steps on one stream
   aspis_round_host(...)                     the same from pinned host memory
   aspis_round_static(copies, d, a, det, out, mode)   the round with no device allocation
+  aspis_sgd(g, w, v, eta, mu)               the model update with the aggregate (Eq. 1, momentum)
 """
 from __future__ import annotations
 
@@ -88,6 +89,7 @@ def _load():
         "aspis_round": ([P, i64, i64, A, P, P, P, P, i32, P, P], i32),
         "aspis_round_host": ([P, P, i64, i64, A, P, P, P, P, i32, P, P, P, P], i32),
         "aspis_round_static": ([P, i64, i64, A, P, i32, P, P], i32),
+        "aspis_sgd": ([P, P, P, i64, ctypes.c_float, ctypes.c_float, P], i32),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -257,6 +259,19 @@ def aspis_round_static(copies, d: int, a: Assignment, det, out, mode: int = MEDI
                                _dev(det, torch.uint8, "det"), mode,
                                _dev(out, torch.float32, "out"), _stream(stream)),
         "aspis_round_static")
+
+
+def aspis_sgd(g, w, v, eta: float, mu: float = 0.9, stream=None):
+    """w, v <- one SGD step with heavy-ball momentum on the aggregate g
+    (in place; see aspis.h).  ``v`` may be None when ``mu == 0``."""
+    import torch
+    n = g.numel()
+    if w.numel() != n or (v is not None and v.numel() != n):
+        raise ValueError("g, w and v must have the same number of elements")
+    vp = None if v is None else _dev(v, torch.float32, "v")
+    _ok(lib.aspis_sgd(_dev(g, torch.float32, "g"), _dev(w, torch.float32, "w"), vp, n,
+                      float(eta), float(mu), _stream(stream)),
+        "aspis_sgd")
 
 
 class RoundBuffers:
