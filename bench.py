@@ -18,7 +18,10 @@ independent replica on its own GPU; there is no data-path collective.
 
 Besides the step, the line reports the model update that follows it
 (aspis_sgd: Eq. 1 with momentum 0.9 on the round's output), timed alone with
-L2 flushed before every launch (key "update"); it is not part of the step.
+L2 flushed before every launch (key "update"), and the clique search on the
+K = 100, r = 5 graphs of the appendix's timing experiment (aspis_detect_wide,
+weak and optimal attacks, q = 5..45; key "table5", beside the paper's
+milliseconds).  Neither is part of the step.
 """
 from __future__ import annotations
 
@@ -39,6 +42,10 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 DEFAULT_CONFIG = "k15_r3_d11m_strong_alie"
+# Table 5: clique enumeration time (ms) in the K = 100, r = 5 graph, NetworkX
+# on an EC2 i3.16xlarge, per number of adversaries q
+TABLE5_MS = {"weak": {5: 9, 15: 7, 25: 5, 35: 5, 45: 5},
+             "optimal": {5: 11, 15: 11, 25: 9, 35: 8, 45: 6}}
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -57,6 +64,8 @@ def parse():
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--no-update", action="store_true",
                    help="skip the separate timing of the model update")
+    p.add_argument("--no-table5", action="store_true",
+                   help="skip the clique-search timing on the K = 100 graphs")
     p.add_argument("--cpu-seconds", type=float, default=12.0,
                    help="target CPU time of the oracle baseline sample")
     return p.parse_args()
@@ -348,6 +357,45 @@ def main():
             del fl
         del wp, vp
 
+    # ---- Table 5: the clique search alone on the K = 100, r = 5 attack graphs
+    table5 = None
+    if not args.no_table5:
+        import numpy as np
+        table5 = {"unit": "ms per search (mean of 20 back-to-back launches, device time)",
+                  "graph": "K=100, r=5 agreement graph of the attack (synth.attack_graph)",
+                  "paper": "NetworkX on EC2 i3.16xlarge (Table 5)", "weak": {}, "optimal": {}}
+        det_w = ap.wide_detection_buffer(dev)
+        det_a = ap.wide_detection_buffer(dev, flags=ap.WIDE_ALL_MAXIMAL)
+        for kind, attack in (("weak", "weak"), ("optimal", "strong")):
+            for q, paper_ms in TABLE5_MS[kind].items():
+                gw = synth.Workload("table5", K=100, r=5, d=1, q=q, attack=attack, seed=q)
+                rows = synth.attack_graph(gw)
+                words = np.array([[(m >> (32 * i)) & 0xFFFFFFFF for i in range(4)] for m in rows],
+                                 dtype=np.uint32)
+                adj = torch.from_numpy(words.view(np.int32)).to(dev)
+                res = {"paper_ms": paper_ms}
+                for key, det_t in (("detect_ms", det_w), ("enumerate_all_ms", det_a)):
+                    with torch.cuda.stream(stream):
+                        for _ in range(3):
+                            ap.aspis_detect_wide(adj, 100, det_t, stream)
+                        e0 = torch.cuda.Event(enable_timing=True)
+                        e1 = torch.cuda.Event(enable_timing=True)
+                        # hold the stream while the host enqueues all 20 launches, so
+                        # the events time the device, not the host's call rate
+                        torch.cuda._sleep(4_000_000)
+                        e0.record(stream)
+                        for _ in range(20):
+                            ap.aspis_detect_wide(adj, 100, det_t, stream)
+                        e1.record(stream)
+                    torch.cuda.synchronize()
+                    res[key] = e0.elapsed_time(e1) / 20
+                dw = ap.DetectionWide.from_tensor(det_a)
+                res.update({"omega": dw.omega, "n_max_cliques": dw.n_max_cliques,
+                            "n_maximal": dw.n_maximal, "search_nodes": dw.search_nodes,
+                            "status": dw.status,
+                            "paper_over_enumerate_all": paper_ms / res["enumerate_all_ms"]})
+                table5[kind][str(q)] = res
+
     # ---- end to end through aspis_round_host from pinned host memory
     e2e = None
     if not args.no_e2e:
@@ -423,6 +471,7 @@ def main():
         "e2e": e2e,
         "cpu_baseline": cpu,
         "update": update,
+        "table5": table5,
     }
     json_line(line)
     if dist:

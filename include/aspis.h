@@ -235,6 +235,52 @@ aspis_status aspis_round_host(const float *host_copies, float *dev_copies,
                               float *dev_out, float *host_out,
                               aspis_detection *host_det, void *stream);
 
+/* ---------------------------------------------------------------------
+ * Detection beyond 32 workers (Algorithm 3 with vertex sets of up to 128
+ * workers).  The round's other steps keep K <= 31; this call takes the
+ * agreement graph directly, as in the clique-timing experiment of the
+ * appendix (Table 5: K = 100, r = 5, whose C(100,5) = 75,287,520 files are
+ * never materialised).  No counterpart of a separate call in the paper. */
+#define ASPIS_WIDE_MAX_K 128
+#define ASPIS_WIDE_ALL_MAXIMAL 1u     /* flags: enumerate every maximal clique */
+
+/* Outcome of aspis_detect_wide; lives in device memory (64 bytes). */
+typedef struct {
+    uint32_t clique_mask[4];     /* the maximum clique with the smallest mask value;
+                                    worker k is bit k % 32 of word k / 32, and word 3
+                                    is the most significant in the comparison */
+    uint64_t n_max_cliques;      /* number of maximum cliques */
+    uint64_t n_maximal;          /* maximal cliques reported: all of them with
+                                    ASPIS_WIDE_ALL_MAXIMAL, else those the size
+                                    bound did not prune (diagnostic) */
+    uint64_t search_nodes;       /* Bron-Kerbosch nodes visited (diagnostic) */
+    int32_t  omega;              /* size of a maximum clique */
+    int32_t  success;            /* 1 iff n_max_cliques == 1 and the search finished */
+    int32_t  status;             /* ASPIS_OK or ASPIS_E_LIMIT */
+    uint32_t node_budget;        /* in: node limit per warp, 0 = 2^20; never written */
+    uint32_t flags;              /* in: ASPIS_WIDE_ALL_MAXIMAL or 0; never written */
+    uint32_t reserved;
+} aspis_detection_wide;
+
+/* All maximum cliques of an agreement graph of K <= 128 workers
+ * (Algorithm 3), by Bron-Kerbosch with Tomita pivoting over 128-bit vertex
+ * sets: one block of four warps splits the root's branches, each warp walks
+ * its branches cooperatively, and workers adjacent to all other candidates
+ * join the clique without branching.  Without flags, branches that cannot
+ * reach the largest clique found so far are pruned (what detection needs);
+ * with
+ * ASPIS_WIDE_ALL_MAXIMAL every maximal clique is enumerated and counted,
+ * as the NetworkX enumeration timed in Table 5 does.
+ *   adj  device [K][4] uint32: row j = the neighbours of worker j, worker k
+ *        at bit k % 32 of word k / 32.  An edge counts only when both rows
+ *        list it; self loops and bits >= K are ignored.
+ *   det  device aspis_detection_wide, in/out (node_budget and flags in)
+ * K < 1 or a NULL pointer returns ASPIS_E_INVAL, K > 128 ASPIS_E_RANGE,
+ * before anything is enqueued.  A warp that exceeds its node budget stops
+ * the search: status = ASPIS_E_LIMIT, success = 0. */
+aspis_status aspis_detect_wide(const uint32_t *adj, int K, aspis_detection_wide *det,
+                               void *stream);
+
 /* The model update that follows the aggregation (Section 2, Eq. 1, with
  * the aggregate of Algorithm 1 in place of the batch gradient), with the
  * heavy-ball momentum of the experiments (Appendix B: momentum 0.9).  For

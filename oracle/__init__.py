@@ -14,6 +14,7 @@ Detection for Distributed Learning"):
 * :func:`pair_agreement`    -- alpha^{(j1,j2)}, Section 4 (second display)
 * :func:`graph`             -- edge iff alpha == C(K-2, r-2), Algorithm 3
 * :func:`max_cliques_brute` / :func:`max_cliques_bk` -- Algorithm 3
+* :func:`max_cliques_wide`  -- Algorithm 3 for up to 128 workers, all maximal cliques counted
 * :func:`select`            -- Algorithm 1, Case 1 / Case 2 (Eq. 2)
 * :func:`aggregate`, :func:`lower_median`, :func:`mean` -- Algorithm 1 updates
 * :func:`sgd`               -- the model update with the aggregate (Eq. 1, momentum)
@@ -71,6 +72,7 @@ def _load():
             lib.oracle_aggregate.argtypes = [P, i64, i32, i64, P, i32, i64, i64, P, i32]
             lib.oracle_lower_median.argtypes = [P, i64, i64, P]
             lib.oracle_mean.argtypes = [P, i64, i64, P]
+            lib.oracle_max_cliques_wide.argtypes = [P, i32, P, P, P, P]
             lib.oracle_sgd.argtypes = [P, P, P, i64, ctypes.c_float, ctypes.c_float]
             _lib = lib
     return _lib
@@ -172,6 +174,41 @@ def max_cliques_bk(adj: np.ndarray, K: int) -> Detection:
     if rc != OK:
         raise ValueError(f"oracle_max_cliques_bk failed: {rc}")
     return Detection(om.value, nm.value, cn.value, calls.value)
+
+
+@dataclass
+class WideDetection:
+    omega: int
+    n_max: int
+    clique: int          # the maximum clique with the smallest mask value, bit k = worker k
+    n_maximal: int       # all maximal cliques
+
+    @property
+    def success(self) -> bool:
+        return self.n_max == 1
+
+
+def max_cliques_wide(adj: np.ndarray, K: int) -> WideDetection:
+    """Algorithm 3 for K <= 128: adj is [K, 4] uint32 (worker k = bit k % 32 of
+    word k // 32); an edge needs both rows to list it."""
+    adj = np.ascontiguousarray(adj, dtype=np.uint32).reshape(K, 4)
+    om, nm, nmax = ctypes.c_int32(), ctypes.c_uint64(), ctypes.c_uint64()
+    canon = np.zeros(4, np.uint32)
+    rc = _load().oracle_max_cliques_wide(_ptr(adj), K, ctypes.byref(om), ctypes.byref(nm),
+                                         _ptr(canon), ctypes.byref(nmax))
+    if rc != OK:
+        raise ValueError(f"oracle_max_cliques_wide failed: {rc}")
+    clique = sum(int(canon[i]) << (32 * i) for i in range(4))
+    return WideDetection(om.value, nm.value, clique, nmax.value)
+
+
+def masks_to_words(rows, K: int) -> np.ndarray:
+    """[K, 4] uint32 adjacency words from K Python-int neighbour masks."""
+    out = np.zeros((K, 4), np.uint32)
+    for j, m in enumerate(rows):
+        for i in range(4):
+            out[j, i] = (int(m) >> (32 * i)) & 0xFFFFFFFF
+    return out
 
 
 def select(file_neq: np.ndarray, a: Assignment, clique: int, success: bool):

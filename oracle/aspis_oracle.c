@@ -17,6 +17,8 @@
  *   oracle_graph               edge rule of G: alpha == C(K-2,r-2) (Section 4, Algorithm 3)
  *   oracle_max_cliques_brute   all maximum cliques by enumerating every vertex subset (Algorithm 3)
  *   oracle_max_cliques_bk      the same by Bron-Kerbosch with pivoting (Tomita et al., cited in Section 4)
+ *   oracle_max_cliques_wide    the same for up to 128 workers, also counting all maximal
+ *                              cliques (the enumeration Table 5 times)
  *   oracle_select              Algorithm 1: Case 1 honest copy / Case 2 majority (Eq. 2)
  *   oracle_lower_median        coordinate-wise median of the chosen gradients (Algorithm 1, Case 2)
  *   oracle_mean                average of the chosen gradients (Algorithm 1, Case 1)
@@ -306,6 +308,115 @@ int oracle_max_cliques_bk(const uint32_t *adj, int K, int32_t *omega,
     *n_max = S.cnt;
     *canon = S.first;
     if (calls) *calls = S.calls;
+    return ORACLE_OK;
+}
+
+/* ------------------------------- Algorithm 3 for up to 128 workers */
+
+/* Vertex sets of up to 128 workers as four 32-bit words: worker k is bit
+ * k % 32 of word k / 32.  A mask's value orders word 3 first. */
+typedef struct {
+    uint32_t w[4];
+} vset;
+
+static int vs_count(vset a)
+{
+    return popcount32(a.w[0]) + popcount32(a.w[1]) + popcount32(a.w[2]) + popcount32(a.w[3]);
+}
+
+static int vs_empty(vset a) { return (a.w[0] | a.w[1] | a.w[2] | a.w[3]) == 0; }
+
+static int vs_has(vset a, int k) { return (int)((a.w[k >> 5] >> (k & 31)) & 1u); }
+
+static vset vs_and(vset a, vset b)
+{
+    for (int i = 0; i < 4; ++i) a.w[i] &= b.w[i];
+    return a;
+}
+
+static vset vs_andnot(vset a, vset b)
+{
+    for (int i = 0; i < 4; ++i) a.w[i] &= ~b.w[i];
+    return a;
+}
+
+static vset vs_with(vset a, int k)
+{
+    a.w[k >> 5] |= 1u << (k & 31);
+    return a;
+}
+
+static vset vs_without(vset a, int k)
+{
+    a.w[k >> 5] &= ~(1u << (k & 31));
+    return a;
+}
+
+static int vs_less(vset a, vset b)
+{
+    for (int i = 3; i >= 0; --i)
+        if (a.w[i] != b.w[i]) return a.w[i] < b.w[i];
+    return 0;
+}
+
+typedef struct {
+    vset adj[128];
+    int K;
+    int best;
+    uint64_t cnt, maximal;
+    vset first;
+} bkw_state;
+
+/* Bron-Kerbosch with Tomita pivoting, as oracle_max_cliques_bk, reporting
+ * every maximal clique R (P and X empty). */
+static void bkw(bkw_state *S, vset R, vset P, vset X)
+{
+    if (vs_empty(P) && vs_empty(X)) {
+        int sz = vs_count(R);
+        S->maximal++;
+        if (sz > S->best) { S->best = sz; S->cnt = 1; S->first = R; }
+        else if (sz == S->best) { S->cnt++; if (vs_less(R, S->first)) S->first = R; }
+        return;
+    }
+    int piv = -1, pbest = -1;
+    for (int u = 0; u < S->K; ++u)
+        if (vs_has(P, u) || vs_has(X, u)) {
+            int c = vs_count(vs_and(P, S->adj[u]));
+            if (c > pbest) { pbest = c; piv = u; }
+        }
+    vset cand = vs_andnot(P, S->adj[piv]);
+    for (int v = 0; v < S->K; ++v) {
+        if (!vs_has(cand, v)) continue;
+        bkw(S, vs_with(R, v), vs_and(P, S->adj[v]), vs_and(X, S->adj[v]));
+        P = vs_without(P, v);
+        X = vs_with(X, v);
+    }
+}
+
+/* adj: [K][4] words, row j = neighbours of worker j.  An edge counts only
+ * when both rows list it; self loops and bits >= K are ignored.  Outputs
+ * omega, the number of maximum cliques, the maximum clique with the smallest
+ * mask value (canon[4]) and the number of maximal cliques. */
+int oracle_max_cliques_wide(const uint32_t *adj, int K, int32_t *omega, uint64_t *n_max,
+                            uint32_t *canon, uint64_t *n_maximal)
+{
+    if (K < 1 || K > 128) return ORACLE_ERANGE;
+    bkw_state *S = (bkw_state *)calloc(1, sizeof(bkw_state));
+    if (!S) return ORACLE_EINVAL;
+    S->K = K;
+    for (int j = 0; j < K; ++j)
+        for (int k = 0; k < K; ++k)
+            if (k != j && ((adj[j * 4 + (k >> 5)] >> (k & 31)) & 1u) &&
+                ((adj[k * 4 + (j >> 5)] >> (j & 31)) & 1u))
+                S->adj[j] = vs_with(S->adj[j], k);
+    vset all = {{0u, 0u, 0u, 0u}}, none = {{0u, 0u, 0u, 0u}};
+    for (int k = 0; k < K; ++k) all = vs_with(all, k);
+    bkw(S, none, all, none);
+    *omega = S->best;
+    *n_max = S->cnt;
+    for (int i = 0; i < 4; ++i) canon[i] = S->first.w[i];
+    *n_maximal = S->maximal;
+    free(S);
     return ORACLE_OK;
 }
 

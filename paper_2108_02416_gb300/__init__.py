@@ -17,6 +17,7 @@ The call names mirror the C entry points:
   aspis_round_host(...)                     the same from pinned host memory
   aspis_round_static(copies, d, a, det, out, mode)   the round with no device allocation
   aspis_sgd(g, w, v, eta, mu)               the model update with the aggregate (Eq. 1, momentum)
+  aspis_detect_wide(adj, K, det)            Algorithm 3 for K <= 128 (graph given directly)
 """
 from __future__ import annotations
 
@@ -66,6 +67,41 @@ class Detection(ctypes.Structure):
 
 DETECTION_BYTES = ctypes.sizeof(Detection)
 
+WIDE_MAX_K = 128
+WIDE_ALL_MAXIMAL = 1
+
+
+class DetectionWide(ctypes.Structure):
+    """Host image of ``aspis_detection_wide`` (64 bytes)."""
+    _fields_ = [("clique_words", ctypes.c_uint32 * 4), ("n_max_cliques", ctypes.c_uint64),
+                ("n_maximal", ctypes.c_uint64), ("search_nodes", ctypes.c_uint64),
+                ("omega", ctypes.c_int32), ("success", ctypes.c_int32),
+                ("status", ctypes.c_int32), ("node_budget", ctypes.c_uint32),
+                ("flags", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
+
+    @classmethod
+    def from_tensor(cls, t):
+        raw = bytes(t.detach().to("cpu").contiguous().numpy().tobytes())
+        return cls.from_buffer_copy(raw)
+
+    @property
+    def clique_mask(self) -> int:
+        """the reported clique as one integer, bit k = worker k"""
+        return sum(int(self.clique_words[i]) << (32 * i) for i in range(4))
+
+
+WIDE_DETECTION_BYTES = ctypes.sizeof(DetectionWide)
+
+
+def wide_detection_buffer(device, node_budget: int = 0, flags: int = 0):
+    """A device uint8 tensor holding an aspis_detection_wide with the inputs set."""
+    import torch
+    d = DetectionWide()
+    d.node_budget = node_budget
+    d.flags = flags
+    host = torch.frombuffer(bytearray(bytes(d)), dtype=torch.uint8)
+    return host.to(device)
+
 
 def _load():
     if not os.path.exists(LIB_PATH):
@@ -90,6 +126,7 @@ def _load():
         "aspis_round_host": ([P, P, i64, i64, A, P, P, P, P, i32, P, P, P, P], i32),
         "aspis_round_static": ([P, i64, i64, A, P, i32, P, P], i32),
         "aspis_sgd": ([P, P, P, i64, ctypes.c_float, ctypes.c_float, P], i32),
+        "aspis_detect_wide": ([P, i32, P, P], i32),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -259,6 +296,20 @@ def aspis_round_static(copies, d: int, a: Assignment, det, out, mode: int = MEDI
                                _dev(det, torch.uint8, "det"), mode,
                                _dev(out, torch.float32, "out"), _stream(stream)),
         "aspis_round_static")
+
+
+def aspis_detect_wide(adj, K: int, det, stream=None):
+    """Algorithm 3 for K <= 128 workers: ``adj`` is a device uint32 [K, 4]
+    tensor (worker k = bit k % 32 of word k // 32), ``det`` a device uint8
+    tensor from :func:`wide_detection_buffer`."""
+    import torch
+    if adj.numel() < 4 * K:
+        raise ValueError("adj must hold K rows of 4 words")
+    if adj.dtype not in (torch.int32, getattr(torch, "uint32", torch.int32)):
+        raise ValueError(f"adj must hold 32-bit words, got {adj.dtype}")
+    _ok(lib.aspis_detect_wide(_dev(adj, None, "adj"), K, _dev(det, torch.uint8, "det"),
+                              _stream(stream)),
+        "aspis_detect_wide")
 
 
 def aspis_sgd(g, w, v, eta: float, mu: float = 0.9, stream=None):

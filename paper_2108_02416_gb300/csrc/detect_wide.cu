@@ -1,0 +1,328 @@
+// Algorithm 3 beyond 32 workers: all maximum cliques of an agreement graph
+// of up to 128 workers, with vertex sets as four 32-bit words.
+//
+// Bron-Kerbosch with Tomita pivoting (pivot = the vertex of P u X with most
+// neighbours in P).  The root's candidates are split over four warps: the
+// k-th candidate c_k starts from R = {c_k}, P = (V minus c_0..c_{k-1}) n N(c_k),
+// X = {c_0..c_{k-1}} n N(c_k), exactly the branch sequential Bron-Kerbosch
+// takes, and warp w takes k = w, w + 4, ...  Each warp walks its branches
+// cooperatively: the current frame (R, P, X, candidates) is the same in all
+// lanes, lane l holds the adjacency rows of workers l, l + 32, l + 64, l + 96
+// in registers, so the pivot is one row-count per lane and a warp max, and
+// parent frames wait on a stack in shared memory (at most K deep: every push
+// adds one worker to R).  Workers of P adjacent to all the rest of P are in
+// every maximal clique of their branch and move to R without branching, so
+// the long chains of nearly complete agreement graphs take one step.  Detection mode prunes a child whose |R| + |P|
+// cannot reach the largest clique any warp has found; enumeration mode
+// (ASPIS_WIDE_ALL_MAXIMAL) prunes nothing and counts every maximal clique.
+// A node budget per warp bounds the search.
+#include "aspis_internal.cuh"
+
+namespace {
+
+constexpr int kMaxK = ASPIS_WIDE_MAX_K;
+constexpr uint32_t kDefaultBudget = 1u << 20;   // nodes per warp
+
+struct VS {
+    uint32_t w[4];
+};
+
+__device__ __forceinline__ VS vs_and(const VS &a, const uint32_t *b)
+{
+    return VS{{a.w[0] & b[0], a.w[1] & b[1], a.w[2] & b[2], a.w[3] & b[3]}};
+}
+
+__device__ __forceinline__ VS vs_andnot(const VS &a, const uint32_t *b)
+{
+    return VS{{a.w[0] & ~b[0], a.w[1] & ~b[1], a.w[2] & ~b[2], a.w[3] & ~b[3]}};
+}
+
+__device__ __forceinline__ int vs_count(const VS &a)
+{
+    return __popc(a.w[0]) + __popc(a.w[1]) + __popc(a.w[2]) + __popc(a.w[3]);
+}
+
+__device__ __forceinline__ int vs_count_and(const VS &a, const VS &b)
+{
+    return __popc(a.w[0] & b.w[0]) + __popc(a.w[1] & b.w[1]) + __popc(a.w[2] & b.w[2]) +
+           __popc(a.w[3] & b.w[3]);
+}
+
+__device__ __forceinline__ bool vs_empty(const VS &a)
+{
+    return (a.w[0] | a.w[1] | a.w[2] | a.w[3]) == 0u;
+}
+
+// index of the lowest member, -1 if empty
+__device__ __forceinline__ int vs_lowest(const VS &a)
+{
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        if (a.w[i]) return 32 * i + __ffs(a.w[i]) - 1;
+    return -1;
+}
+
+// (word selected by comparison, not by index, so sets stay in registers)
+__device__ __forceinline__ void vs_set(VS &a, int k)
+{
+#pragma unroll
+    for (int i = 0; i < 4; ++i) a.w[i] |= (k >> 5) == i ? 1u << (k & 31) : 0u;
+}
+
+__device__ __forceinline__ void vs_clear(VS &a, int k)
+{
+#pragma unroll
+    for (int i = 0; i < 4; ++i) a.w[i] &= (k >> 5) == i ? ~(1u << (k & 31)) : 0xffffffffu;
+}
+
+// a < b as 128-bit numbers, word 3 most significant
+__device__ __forceinline__ bool vs_less(const VS &a, const VS &b)
+{
+#pragma unroll
+    for (int i = 3; i >= 0; --i)
+        if (a.w[i] != b.w[i]) return a.w[i] < b.w[i];
+    return false;
+}
+
+constexpr int kWarps = 4;
+
+__global__ void __launch_bounds__(kWarps * 32)
+detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wide *det)
+{
+    __shared__ uint32_t raw[kMaxK][4];
+    __shared__ uint32_t adj[kMaxK][4];
+    __shared__ uint32_t stack[kWarps][kMaxK][16];      // R, P, X, C of waiting parents
+    __shared__ int shared_best;
+    __shared__ int w_best[kWarps], w_over[kWarps];
+    __shared__ unsigned long long w_count[kWarps], w_maximal[kWarps], w_nodes[kWarps];
+    __shared__ uint32_t w_first[kWarps][4];
+    const int tid = threadIdx.x, lane = tid & 31, wp = tid >> 5;
+    const unsigned full = 0xffffffffu;
+    for (int i = tid; i < kMaxK * 4; i += kWarps * 32) raw[i >> 2][i & 3] = (i >> 2) < K ? adj_g[i] : 0u;
+    if (tid == 0) shared_best = 0;
+    __syncthreads();
+    // symmetric part: bit k of row j iff both rows list the edge; no self
+    // loops, nothing at or beyond K
+    for (int j = tid; j < kMaxK; j += kWarps * 32) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            uint32_t m = 0u;
+            uint32_t x = j < K ? raw[j][i] : 0u;
+            while (x) {
+                const int b = __ffs(x) - 1;
+                x &= x - 1u;
+                const int k = 32 * i + b;
+                if (k < K && k != j && ((raw[k][j >> 5] >> (j & 31)) & 1u)) m |= 1u << b;
+            }
+            adj[j][i] = m;
+        }
+    }
+    __syncthreads();
+
+    const uint32_t budget = det->node_budget ? det->node_budget : kDefaultBudget;
+    const bool all = (det->flags & ASPIS_WIDE_ALL_MAXIMAL) != 0u;
+    // this lane's rows: workers lane + 32 j
+    const VS own0{{adj[lane][0], adj[lane][1], adj[lane][2], adj[lane][3]}};
+    const VS own1{{adj[lane + 32][0], adj[lane + 32][1], adj[lane + 32][2], adj[lane + 32][3]}};
+    const VS own2{{adj[lane + 64][0], adj[lane + 64][1], adj[lane + 64][2], adj[lane + 64][3]}};
+    const VS own3{{adj[lane + 96][0], adj[lane + 96][1], adj[lane + 96][2], adj[lane + 96][3]}};
+
+    int best = 0;
+    uint64_t count = 0, maximal = 0, nodes = 0;
+    VS first{{0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu}};
+    bool over = false;
+    bool live = true;           // false while every warp settles the same root frame
+    auto report = [&](const VS R) {
+        if (!live) return;
+        const int sz = vs_count(R);
+        ++maximal;
+        if (sz > best) {
+            best = sz;
+            count = 1;
+            first = R;
+            if (lane == 0) atomicMax(&shared_best, sz);
+        } else if (sz == best) {
+            ++count;
+            if (vs_less(R, first)) first = R;
+        }
+    };
+
+    // Settles a new frame (R, P, X).  Workers of P adjacent to all the rest
+    // of P lie in every maximal clique of the branch, so they move to R at
+    // once (X keeps only their common neighbours); when P is a clique that
+    // leaves P empty, and R is maximal iff X is empty.  Returns true with
+    // the candidates C = P minus the pivot's neighbours when the frame must
+    // be branched, false when it is finished (reported or pruned).  Every
+    // pass of the loop moves at least one worker out of P.
+    auto settle = [&](VS &R, VS &P, VS &X, VS &C) -> bool {
+        while (true) {
+            if (vs_empty(P)) {
+                if (vs_empty(X)) report(R);
+                return false;
+            }
+            if (!all) {
+                const int bound = max(best, *(volatile int *)&shared_best);
+                if (vs_count(R) + vs_count(P) < bound) return false;
+            }
+            const uint32_t np1 = (uint32_t)vs_count(P);          // |P|; a universal worker has |P| - 1
+            uint32_t key = 0u;
+            VS U{{0u, 0u, 0u, 0u}};
+            VS common{{0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu}};
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int u = lane + 32 * j;
+                const bool inP = (P.w[j] >> lane) & 1u, inX = (X.w[j] >> lane) & 1u;
+                const VS &oj = j == 0 ? own0 : j == 1 ? own1 : j == 2 ? own2 : own3;
+                uint32_t c = 0u;
+                if (inP || inX) {
+                    c = (uint32_t)vs_count_and(P, oj);
+                    key = max(key, ((c + 1u) << 8) | (uint32_t)(255 - u));
+                }
+                const bool uni = inP && c + 1u == np1;
+                U.w[j] = __ballot_sync(full, uni);
+                if (uni) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) common.w[i] &= oj.w[i];
+                }
+            }
+            if (!vs_empty(U)) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    common.w[i] = __reduce_and_sync(full, common.w[i]);
+                    R.w[i] |= U.w[i];
+                    P.w[i] &= ~U.w[i];
+                    X.w[i] &= common.w[i];
+                }
+                continue;
+            }
+            // pivot: the worker of P u X with most neighbours in P, lowest
+            // index on ties (any pivot enumerates the same cliques)
+            key = __reduce_max_sync(full, key);
+            const int piv = 255 - (int)(key & 255u);      // P is not empty, so key != 0
+            C = vs_andnot(P, adj[piv]);
+            return true;
+        }
+    };
+
+    // the root frame, settled by every warp alike (reports counted once)
+    VS R0{{0u, 0u, 0u, 0u}}, P0{{0u, 0u, 0u, 0u}}, X0{{0u, 0u, 0u, 0u}}, C0{{0u, 0u, 0u, 0u}};
+    for (int v = 0; v < K; ++v) vs_set(P0, v);
+    live = wp == 0;
+    const bool branch0 = settle(R0, P0, X0, C0);
+    live = true;
+    if (!branch0) C0 = VS{{0u, 0u, 0u, 0u}};
+    int k = 0;
+    while (!over) {
+        const int ck = vs_lowest(C0);
+        if (ck < 0) break;
+        vs_clear(C0, ck);
+        const bool mine = (k++ % kWarps) == wp;
+        // branch c_k: R, P and X as sequential Bron-Kerbosch leaves them
+        VS R = R0, P = vs_and(P0, adj[ck]), X = vs_and(X0, adj[ck]), C;
+        vs_set(R, ck);
+        vs_clear(P0, ck);
+        vs_set(X0, ck);
+        if (!mine) continue;
+        if (++nodes > budget) {
+            over = true;
+            break;
+        }
+        if (!settle(R, P, X, C)) continue;
+        int sp = 0;
+        while (true) {
+            const int u = vs_lowest(C);
+            if (u < 0) {
+                if (sp == 0) break;
+                --sp;                                   // back to the parent
+                __syncwarp();
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    R.w[i] = stack[wp][sp][i];
+                    P.w[i] = stack[wp][sp][4 + i];
+                    X.w[i] = stack[wp][sp][8 + i];
+                    C.w[i] = stack[wp][sp][12 + i];
+                }
+                __syncwarp();
+                continue;
+            }
+            if (++nodes > budget) {
+                over = true;
+                break;
+            }
+            vs_clear(C, u);
+            VS Ru = R, Cu;
+            vs_set(Ru, u);
+            VS Pu = vs_and(P, adj[u]);
+            VS Xu = vs_and(X, adj[u]);
+            vs_clear(P, u);
+            vs_set(X, u);
+            if (!settle(Ru, Pu, Xu, Cu)) continue;
+            if (sp >= kMaxK) {                          // unreachable: |R| grows by one per frame
+                over = true;
+                break;
+            }
+            // the parent waits on the stack; the child becomes the frame
+            if (lane < 16) {
+                uint32_t val = 0u;
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    if ((lane & 3) == i) val = lane < 4 ? R.w[i] : lane < 8 ? P.w[i] : lane < 12 ? X.w[i] : C.w[i];
+                stack[wp][sp][lane] = val;
+            }
+            __syncwarp();
+            ++sp;
+            R = Ru;
+            P = Pu;
+            X = Xu;
+            C = Cu;
+        }
+    }
+
+    // reduction over warps: omega, maximum cliques of that size, the smallest
+    if (lane == 0) {
+        w_best[wp] = best;
+        w_over[wp] = over ? 1 : 0;
+        w_count[wp] = count;
+        w_maximal[wp] = maximal;
+        w_nodes[wp] = nodes;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) w_first[wp][i] = count ? first.w[i] : 0xffffffffu;
+    }
+    __syncthreads();
+    if (tid == 0) {
+        int omega = 0;
+        for (int q = 0; q < kWarps; ++q) omega = max(omega, w_best[q]);
+        uint64_t n = 0, nmx = 0, nds = 0;
+        bool any_over = false;
+        VS c{{0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu}};
+        for (int q = 0; q < kWarps; ++q) {
+            nmx += w_maximal[q];
+            nds += w_nodes[q];
+            any_over |= w_over[q] != 0;
+            if (w_best[q] == omega && w_count[q]) {
+                n += w_count[q];
+                const VS f{{w_first[q][0], w_first[q][1], w_first[q][2], w_first[q][3]}};
+                if (vs_less(f, c)) c = f;
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) det->clique_mask[i] = c.w[i];
+        det->n_max_cliques = n;
+        det->n_maximal = nmx;
+        det->search_nodes = nds;
+        det->omega = omega;
+        det->success = (n == 1u && !any_over) ? 1 : 0;
+        det->status = any_over ? ASPIS_E_LIMIT : ASPIS_OK;
+    }
+}
+
+}  // namespace
+
+extern "C" aspis_status aspis_detect_wide(const uint32_t *adj, int K, aspis_detection_wide *det,
+                                          void *stream)
+{
+    if (!adj || !det || K < 1) return ASPIS_E_INVAL;
+    if (K > ASPIS_WIDE_MAX_K) return ASPIS_E_RANGE;
+    detect_wide_kernel<<<1, kWarps * 32, 0, (cudaStream_t)stream>>>(adj, K, det);
+    return cudaGetLastError() == cudaSuccess ? ASPIS_OK : ASPIS_E_CUDA;
+}

@@ -200,6 +200,43 @@ def corrupted_mask(w: Workload, file_workers: np.ndarray) -> np.ndarray:
     return mask
 
 
+def attack_graph(w: Workload) -> list[int]:
+    """Neighbour masks (bit k = worker k) of the agreement graph that the
+    workload's attack leaves, for any K, without materialising the C(K,r)
+    files: an edge (j, k) is missing iff some file held by both carries
+    different copies from j and k.
+      weak / all_alie: every copy an adversary holds is distorted, the same
+        way by all colluders, so exactly the adversary-honest pairs disagree.
+      strong: adversary a and worker k of D disagree iff some file inside
+        A u D holds both and at least r' = (r+1)/2 adversaries; all other
+        pairs agree (adversaries return honest copies elsewhere).
+    Used for graph-only workloads (the clique search alone, as in the
+    K = 100 timing experiment); for small K the tests check it against the
+    graph computed from actual copies."""
+    A, D = adversary_sets(w)
+    K, r = w.K, w.r
+    missing = set()
+    if A and w.attack in ("all_alie", "weak"):
+        H = [k for k in range(K) if k not in set(A)]
+        missing = {(a, h) for a in A for h in H}
+    elif A and w.attack == "strong":
+        rp = (r + 1) // 2
+        q_a, q_d = len(A), len(D)
+        # the r - 2 other members: x more adversaries (x >= r' - 1) and
+        # r - 2 - x more workers of D
+        ok = any(rp - 1 <= x <= q_a - 1 and 0 <= r - 2 - x <= q_d - 1 for x in range(r - 1))
+        if ok:
+            missing = {(a, k) for a in A for k in D}
+    elif A:
+        raise ValueError(w.attack)
+    rows = [0] * K
+    for j in range(K):
+        for k in range(K):
+            if j != k and (j, k) not in missing and (k, j) not in missing:
+                rows[j] |= 1 << k
+    return rows
+
+
 def _alie_np(w: Workload, c0: int, c1: int) -> np.ndarray:
     b = 0.01 * normal_np(w.seed, STREAM_B, c0, c1)
     f = w.f
