@@ -281,6 +281,38 @@ typedef struct {
 aspis_status aspis_detect_wide(const uint32_t *adj, int K, aspis_detection_wide *det,
                                void *stream);
 
+/* The round for copies that are not bit-identical.  Section 5 (after
+ * Algorithm 1) notes that honest copies differing by floating-point effects
+ * can be handled: Case 1 averages the honest copies of each file, Case 2
+ * clusters the copies and averages the largest cluster.  Readings:
+ *   - copies a, b of a file are close iff |a[c] - b[c]| <= tau for every
+ *     c < d (difference and magnitude in fp32; never close where either is
+ *     NaN); the graph rule uses "close" for "equal";
+ *   - Case 1 averages the slots whose worker is in the clique (a file with
+ *     none is dropped); Case 2 the largest connected component of "close"
+ *     among the r slots, ties to the component holding the lower slot;
+ *   - the average of the chosen copies x_s, x0 the first: e_s = 0 where x_s
+ *     equals x0 bitwise, else fp32(x_s - x0); acc = fp32 sum of the e_s in
+ *     slot order; mean = x0 if acc == 0, else fp32(x0 + fp32(acc / k)).
+ *     Identical copies give their common value exactly.
+ * The lower median (mode 0) or mean (mode 1) of the kept files' averages is
+ * written to out.  With tau = 0 and copies without NaNs or signed-zero
+ * differences the result equals aspis_round's.
+ *   tau        >= 0 (NaN or negative: ASPIS_E_INVAL)
+ *   file_neq, adj, det   as for aspis_round ("not close" bits)
+ *   slot_mask  device [f] uint8, out: the slots averaged for file i (0 = dropped)
+ *   sel        device [f] int8, out: 0 for kept files, -1 for dropped ones
+ *   means      device [f][ldm] fp32, out: the averages (rows of dropped
+ *              files untouched); ldm >= d; 16-byte aligned with ldm % 4 == 0
+ *              for the 128-bit path
+ * Reads f*r*d*4 bytes (compare) plus the chosen copies (averages), writes
+ * n_kept*d*4 and reads them again (median).  f must be <= ASPIS_MAX_AGG_FILES. */
+aspis_status aspis_round_tolerant(const float *copies, int64_t d, int64_t ld,
+                                  const aspis_assignment *a, float tau, uint32_t *file_neq,
+                                  uint32_t *adj, aspis_detection *det, uint8_t *slot_mask,
+                                  int8_t *sel, float *means, int64_t ldm, int mode, float *out,
+                                  void *stream);
+
 /* The model update that follows the aggregation (Section 2, Eq. 1, with
  * the aggregate of Algorithm 1 in place of the batch gradient), with the
  * heavy-ball momentum of the experiments (Appendix B: momentum 0.9).  For

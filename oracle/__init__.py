@@ -18,6 +18,8 @@ Detection for Distributed Learning"):
 * :func:`select`            -- Algorithm 1, Case 1 / Case 2 (Eq. 2)
 * :func:`aggregate`, :func:`lower_median`, :func:`mean` -- Algorithm 1 updates
 * :func:`sgd`               -- the model update with the aggregate (Eq. 1, momentum)
+* :func:`run_round_tolerant` -- the variant for copies that are not bit-identical
+  (Section 5: average the honest copies / the largest cluster)
 * :func:`run_round`         -- the whole step in the paper's order
 """
 from __future__ import annotations
@@ -74,6 +76,10 @@ def _load():
             lib.oracle_mean.argtypes = [P, i64, i64, P]
             lib.oracle_max_cliques_wide.argtypes = [P, i32, P, P, P, P]
             lib.oracle_sgd.argtypes = [P, P, P, i64, ctypes.c_float, ctypes.c_float]
+            lib.oracle_file_agreement_tol.argtypes = [P, i64, i32, i64, i64, ctypes.c_float, P, i32]
+            lib.oracle_select_tol.argtypes = [P, P, i64, i32, ctypes.c_uint32, i32, P]
+            lib.oracle_select_tol.restype = i64
+            lib.oracle_file_means.argtypes = [P, i64, i32, i64, i64, P, P]
             _lib = lib
     return _lib
 
@@ -307,3 +313,73 @@ def run_round(copies: np.ndarray, a: Assignment, d: int | None = None, mode: int
     if aggregate_out and n_sel > 0:
         out = aggregate(copies, sel, mode, 0, d, nthreads)
     return RoundResult(file_neq, alpha, adj, det, sel, n_sel, out)
+
+
+# ------------------------------------------------ copies that are not bit-identical
+
+def file_agreement_tol(copies: np.ndarray, tau: float, d: int | None = None,
+                       nthreads=None) -> np.ndarray:
+    """Per-file mismatch words under the tolerance: bit p set iff the copies
+    of slot pair p are not within tau on every coordinate (fp32)."""
+    copies = np.ascontiguousarray(copies, dtype=np.float32)
+    f, r, ld = copies.shape
+    d = ld if d is None else d
+    out = np.zeros(max(f, 1), np.uint32)
+    rc = _load().oracle_file_agreement_tol(_ptr(copies), f, r, d, ld, float(np.float32(tau)),
+                                           _ptr(out), _threads(nthreads))
+    if rc != OK:
+        raise ValueError(f"oracle_file_agreement_tol failed: {rc}")
+    return out[:f]
+
+
+def select_tol(file_neq: np.ndarray, a: Assignment, clique: int, success: bool):
+    """(slot_mask[f] uint8, files kept): the copies averaged for each file."""
+    file_neq = np.ascontiguousarray(file_neq, dtype=np.uint32)
+    fw = np.ascontiguousarray(a.file_workers, dtype=np.uint8)
+    mask = np.zeros(max(a.f, 1), np.uint8)
+    n = _load().oracle_select_tol(_ptr(file_neq), _ptr(fw), a.f, a.r, ctypes.c_uint32(clique),
+                                  1 if success else 0, _ptr(mask))
+    return mask[: a.f], int(n)
+
+
+def file_means(copies: np.ndarray, slot_mask: np.ndarray, d: int | None = None) -> np.ndarray:
+    """[f, d] averages of the chosen copies of every file (zeros where dropped)."""
+    copies = np.ascontiguousarray(copies, dtype=np.float32)
+    f, r, ld = copies.shape
+    d = ld if d is None else d
+    mask = np.ascontiguousarray(slot_mask, dtype=np.uint8)
+    out = np.zeros((max(f, 1), max(d, 1)), np.float32)
+    rc = _load().oracle_file_means(_ptr(copies), f, r, d, ld, _ptr(mask), _ptr(out))
+    if rc != OK:
+        raise ValueError(f"oracle_file_means failed: {rc}")
+    return out[:f, :d]
+
+
+@dataclass
+class TolerantResult:
+    file_neq: np.ndarray
+    adj: np.ndarray
+    det: Detection
+    slot_mask: np.ndarray
+    n_kept: int
+    means: np.ndarray
+    out: np.ndarray | None
+
+
+def run_round_tolerant(copies: np.ndarray, a: Assignment, tau: float, d: int | None = None,
+                       mode: int = 0, nthreads=None) -> TolerantResult:
+    """The round with "close within tau" in place of bitwise equality; the
+    kept files' averaged copies are reduced by the lower median (mode 0) or
+    the mean (mode 1)."""
+    f, r, ld = copies.shape
+    d = ld if d is None else d
+    file_neq = file_agreement_tol(copies, tau, d, nthreads)
+    adj = graph(pair_agreement(file_neq, a), a.K, a.r)
+    det = detect(adj, a.K)
+    mask, n = select_tol(file_neq, a, det.clique, det.success)
+    means = file_means(copies, mask, d)
+    out = None
+    if n > 0:
+        kept = means[mask != 0]
+        out = lower_median(kept) if mode == 0 else mean(kept)
+    return TolerantResult(file_neq, adj, det, mask, n, means, out)

@@ -24,6 +24,10 @@
  *   oracle_mean                average of the chosen gradients (Algorithm 1, Case 1)
  *   oracle_sgd                 the model update with the aggregate (Section 2, Eq. 1;
  *                              Algorithm 1), with heavy-ball momentum (Appendix B)
+ *   oracle_file_agreement_tol, oracle_select_tol, oracle_file_means
+ *                              the variant for copies that are not bit-identical
+ *                              (Section 5, after Algorithm 1: average the honest
+ *                              copies, or the largest cluster of copies)
  *
  * Readings where the paper is silent (each also listed in the design notes):
  *   - file i <-> the i-th r-subset of workers in lexicographic order; Example 1
@@ -130,6 +134,7 @@ typedef struct {
     const float *copies;
     int64_t f0, f1, d, ld;
     int r;
+    float tau;                 /* tolerant variant only */
     uint32_t *file_neq;
 } agree_job;
 
@@ -606,6 +611,144 @@ int oracle_sgd(const float *g, float *w, float *v, int64_t m, float eta, float m
             w[c] = fmaf(-eta, v[c], w[c]);
         } else {
             w[c] = fmaf(-eta, g[c], w[c]);
+        }
+    }
+    return ORACLE_OK;
+}
+
+/* --------------------------------- copies that are not bit-identical */
+
+/* Section 5 (after Algorithm 1) notes that honest copies differing by
+ * floating-point effects can still be handled: in Case 1 the PS averages
+ * the honest copies of a file, in Case 2 it clusters the copies and
+ * averages the largest cluster.  Readings, which the paper leaves open:
+ *   - copies a, b of a file are close iff |a[c] - b[c]| <= tau for every
+ *     c < d, the difference and its magnitude in fp32 (never close where
+ *     either value is NaN); the graph and clique steps use "close" for
+ *     "equal";
+ *   - clusters are the connected components of "close" among the r slots;
+ *     the largest wins, ties to the one holding the lower slot;
+ *   - the average of the chosen copies x_s (x0 the first) per coordinate:
+ *     deviations e_s = 0 where x_s equals x0 bitwise, else fp32(x_s - x0);
+ *     acc = fp32 sum of e_s in slot order; the mean is x0 when acc == 0,
+ *     else fp32(x0 + fp32(acc / k)).  Identical copies give their common
+ *     value exactly (also -0, infinities and NaNs). */
+
+static void *agree_tol_worker(void *arg)
+{
+    agree_job *J = (agree_job *)arg;
+    const float tau = J->tau;
+    for (int64_t i = J->f0; i < J->f1; ++i) {
+        uint32_t w = 0;
+        for (int s = 0; s < J->r; ++s)
+            for (int t = s + 1; t < J->r; ++t) {
+                const float *a = J->copies + (i * J->r + s) * J->ld;
+                const float *b = J->copies + (i * J->r + t) * J->ld;
+                int close = 1;
+                for (int64_t c = 0; c < J->d && close; ++c) {
+                    float diff = a[c] - b[c];
+                    if (!(fabsf(diff) <= tau)) close = 0;
+                }
+                if (!close) w |= 1u << pair_bit(J->r, s, t);
+            }
+        J->file_neq[i] = w;
+    }
+    return NULL;
+}
+
+/* file_neq[i] bit pair_bit(s,t) is 1 iff copies s and t of file i are not
+ * close.  tau must be >= 0 (a NaN tau is rejected). */
+int oracle_file_agreement_tol(const float *copies, int64_t f, int r, int64_t d, int64_t ld,
+                              float tau, uint32_t *file_neq, int nthreads)
+{
+    if (r < 2 || r > 8 || d < 0 || ld < d || f < 0 || !(tau >= 0.0f)) return ORACLE_EINVAL;
+    if (nthreads < 1) nthreads = 1;
+    if (nthreads > 256) nthreads = 256;
+    pthread_t th[256];
+    agree_job jobs[256];
+    for (int t = 0; t < nthreads; ++t) {
+        jobs[t].copies = copies;
+        jobs[t].f0 = f * t / nthreads;
+        jobs[t].f1 = f * (t + 1) / nthreads;
+        jobs[t].d = d;
+        jobs[t].ld = ld;
+        jobs[t].r = r;
+        jobs[t].tau = tau;
+        jobs[t].file_neq = file_neq;
+        pthread_create(&th[t], NULL, agree_tol_worker, &jobs[t]);
+    }
+    for (int t = 0; t < nthreads; ++t) pthread_join(th[t], NULL);
+    return ORACLE_OK;
+}
+
+/* slot_mask[i] = the slots whose copies are averaged for file i (bit s =
+ * slot s), 0 when the file is dropped.  Case 1 (success): the slots whose
+ * worker is in the clique.  Case 2: the largest cluster.  Returns the
+ * number of files kept. */
+int64_t oracle_select_tol(const uint32_t *file_neq, const uint8_t *file_workers, int64_t f,
+                          int r, uint32_t clique, int success, uint8_t *slot_mask)
+{
+    int64_t kept = 0;
+    for (int64_t i = 0; i < f; ++i) {
+        uint32_t m = 0;
+        if (success) {
+            for (int s = 0; s < r; ++s)
+                if ((clique >> file_workers[i * r + s]) & 1u) m |= 1u << s;
+        } else {
+            int comp[8];
+            for (int s = 0; s < r; ++s) comp[s] = s;
+            /* union of close pairs, repeated until no label changes */
+            for (int changed = 1; changed;) {
+                changed = 0;
+                for (int s = 0; s < r; ++s)
+                    for (int t = s + 1; t < r; ++t)
+                        if (!((file_neq[i] >> pair_bit(r, s, t)) & 1u) && comp[s] != comp[t]) {
+                            int lo = comp[s] < comp[t] ? comp[s] : comp[t];
+                            int hi = comp[s] < comp[t] ? comp[t] : comp[s];
+                            for (int u = 0; u < r; ++u)
+                                if (comp[u] == hi) comp[u] = lo;
+                            changed = 1;
+                        }
+            }
+            int best = -1, best_size = 0;
+            for (int s = 0; s < r; ++s) {       /* labels are each component's lowest slot */
+                if (comp[s] != s) continue;
+                int size = 0;
+                for (int u = 0; u < r; ++u) size += comp[u] == s;
+                if (size > best_size) { best_size = size; best = s; }
+            }
+            for (int u = 0; u < r; ++u)
+                if (comp[u] == best) m |= 1u << u;
+        }
+        slot_mask[i] = (uint8_t)m;
+        if (m) ++kept;
+    }
+    return kept;
+}
+
+/* means[i*d + c] = the average of the copies in slot_mask[i] (reading
+ * above); files with an empty mask are left untouched. */
+int oracle_file_means(const float *copies, int64_t f, int r, int64_t d, int64_t ld,
+                      const uint8_t *slot_mask, float *means)
+{
+    if (r < 1 || r > 8 || d < 0 || ld < d || f < 0) return ORACLE_EINVAL;
+    for (int64_t i = 0; i < f; ++i) {
+        const uint32_t m = slot_mask[i];
+        if (!m) continue;
+        int k = 0, s0 = -1;
+        for (int s = 0; s < r; ++s)
+            if ((m >> s) & 1u) { if (s0 < 0) s0 = s; ++k; }
+        const float *x0 = copies + (i * r + s0) * ld;
+        for (int64_t c = 0; c < d; ++c) {
+            float acc = 0.0f;
+            for (int s = 0; s < r; ++s) {
+                if (!((m >> s) & 1u)) continue;
+                const float xs = copies[(i * r + s) * ld + c];
+                float e = 0.0f;
+                if (memcmp(&xs, &x0[c], 4) != 0) e = xs - x0[c];
+                acc = acc + e;
+            }
+            means[i * d + c] = acc == 0.0f ? x0[c] : x0[c] + acc / (float)k;
         }
     }
     return ORACLE_OK;

@@ -18,6 +18,7 @@ The call names mirror the C entry points:
   aspis_round_static(copies, d, a, det, out, mode)   the round with no device allocation
   aspis_sgd(g, w, v, eta, mu)               the model update with the aggregate (Eq. 1, momentum)
   aspis_detect_wide(adj, K, det)            Algorithm 3 for K <= 128 (graph given directly)
+  aspis_round_tolerant(copies, d, a, tau, ...)   the round for copies that are not bit-identical
 """
 from __future__ import annotations
 
@@ -127,6 +128,8 @@ def _load():
         "aspis_round_static": ([P, i64, i64, A, P, i32, P, P], i32),
         "aspis_sgd": ([P, P, P, i64, ctypes.c_float, ctypes.c_float, P], i32),
         "aspis_detect_wide": ([P, i32, P, P], i32),
+        "aspis_round_tolerant": ([P, i64, i64, A, ctypes.c_float, P, P, P, P, P, P, i64, i32, P, P],
+                                 i32),
     }
     for name, (args, res) in sig.items():
         fn = getattr(lib, name)
@@ -312,6 +315,24 @@ def aspis_detect_wide(adj, K: int, det, stream=None):
         "aspis_detect_wide")
 
 
+def aspis_round_tolerant(copies, d: int, a: Assignment, tau: float, file_neq, adj, det, slot_mask,
+                         sel, means, out, mode: int = MEDIAN, stream=None):
+    """The round with "close within tau" in place of bitwise equality and the
+    kept files' averaged copies aggregated (see aspis.h).  ``means`` is a
+    device float32 [f, ldm] tensor with ldm >= d."""
+    import torch
+    ld = _ld(copies, a)
+    if means.dim() != 2 or means.shape[0] != a.f or means.shape[1] < d:
+        raise ValueError(f"means must be [f={a.f}, ldm >= d], got {tuple(means.shape)}")
+    _ok(lib.aspis_round_tolerant(_dev(copies, torch.float32, "copies"), d, ld, a.ref, float(tau),
+                                 _dev(file_neq, torch.int32, "file_neq"), _dev(adj, torch.int32, "adj"),
+                                 _dev(det, torch.uint8, "det"), _dev(slot_mask, torch.uint8, "slot_mask"),
+                                 _dev(sel, torch.int8, "sel"), _dev(means, torch.float32, "means"),
+                                 int(means.shape[1]), mode, _dev(out, torch.float32, "out"),
+                                 _stream(stream)),
+        "aspis_round_tolerant")
+
+
 def aspis_sgd(g, w, v, eta: float, mu: float = 0.9, stream=None):
     """w, v <- one SGD step with heavy-ball momentum on the aggregate g
     (in place; see aspis.h).  ``v`` may be None when ``mu == 0``."""
@@ -338,3 +359,14 @@ class RoundBuffers:
 
     def detection(self) -> Detection:
         return Detection.from_tensor(self.det)
+
+
+class TolerantBuffers(RoundBuffers):
+    """RoundBuffers plus the slot masks and the [f, round_up(d, 4)] averages
+    of the tolerant round."""
+
+    def __init__(self, a: Assignment, d: int, device):
+        import torch
+        super().__init__(a, d, device)
+        self.slot_mask = torch.zeros(a.f, dtype=torch.uint8, device=device)
+        self.means = torch.zeros((a.f, (d + 3) // 4 * 4), dtype=torch.float32, device=device)

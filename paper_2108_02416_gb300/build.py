@@ -18,7 +18,8 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libaspis.so")
 SOURCES = ["assign.cpp", "api.cu", "check.cu", "detect.cu", "aggregate.cu",
-           "round_static.cu", "update.cu", "detect_wide.cu"]
+           "round_static.cu", "update.cu", "detect_wide.cu",
+           "tolerant.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -18,8 +18,11 @@ workers and r = 3; synthetic vectors stand in for the gradients):
   n_f[c] = 0.001 * z_f[c]                (per-file noise)
   g_f[c] = fp32(b[c] + n_f[c])           (all honest copies of file f are g_f)
 Distortions (Section 6.1): ALIE fp32(mean_f g - z * std_f g) (population std,
-double, file order); reversed gradient fp32(-c * g_f).  Colluding adversaries
-return identical corrupted vectors.
+double, file order); reversed gradient fp32(-c * g_f); Fall of Empires (inner
+product manipulation) fp32(-z * mean_f g).  Colluding adversaries return
+identical corrupted vectors.  For the variant with copies that are not
+bit-identical, copy_noise > 0 gives honest copy (i, s) the value
+fp32(g_i + copy_noise * z_{i,s}) instead of g_i.
 """
 from __future__ import annotations
 
@@ -36,6 +39,7 @@ C2 = 0x94D049BB133111EB
 STREAM_B = 0
 STREAM_PERM = 1
 STREAM_FILE0 = 16
+STREAM_COPY0 = 1 << 40          # + 8 i + s: per-copy noise of honest copies
 
 
 def _mix64_int(z: int) -> int:
@@ -131,7 +135,9 @@ class Workload:
       "strong"        optimal attack of Theorem 1: A and a disagreement set D
                       (both random by seed); an adversary corrupts its copy of
                       file F iff F is inside A u D and |F n A| >= r' = (r+1)/2
-    distortion: "alie" (z) or "reversed" (scale)
+    distortion: "alie" (z), "foe" (z = the Fall-of-Empires epsilon) or
+      "reversed" (scale)
+    copy_noise: std of the per-copy noise of honest copies (0 = bit-identical)
     """
     name: str
     K: int
@@ -145,6 +151,7 @@ class Workload:
     seed: int = 0
     adversaries: Sequence[int] | None = None
     ld_align: int = 32
+    copy_noise: float = 0.0
     extra: dict = field(default_factory=dict)
 
     @property
@@ -244,6 +251,8 @@ def _alie_np(w: Workload, c0: int, c1: int) -> np.ndarray:
     for i in range(f):
         s += honest_np(w.seed, i, c0, c1, b).astype(np.float64)
     mu = s / f
+    if w.distortion == "foe":
+        return (-w.z * mu).astype(np.float32)
     v = np.zeros(c1 - c0)
     for i in range(f):
         t = honest_np(w.seed, i, c0, c1, b).astype(np.float64) - mu
@@ -260,6 +269,8 @@ def _alie_torch(w: Workload, c0: int, c1: int, device):
     for i in range(f):
         s += honest_torch(w.seed, i, c0, c1, device, b).to(torch.float64)
     mu = s / f
+    if w.distortion == "foe":
+        return (-w.z * mu).to(torch.float32)
     v = torch.zeros_like(s)
     for i in range(f):
         t = honest_torch(w.seed, i, c0, c1, device, b).to(torch.float64) - mu
@@ -283,15 +294,19 @@ def build_copies_np(w: Workload, file_workers: np.ndarray, c0: int = 0,
     out = np.full((f, r, width), pad_value, np.float32)
     mask = corrupted_mask(w, fw)
     bad = None
-    if mask.any() and w.distortion == "alie":
+    if mask.any() and w.distortion in ("alie", "foe"):
         bad = _alie_np(w, c0, c1)
     b = 0.01 * normal_np(w.seed, STREAM_B, c0, c1)
     for i in range(f):
         g = honest_np(w.seed, i, c0, c1, b)
         for s in range(r):
             if not mask[i, s]:
-                out[i, s, : c1 - c0] = g
-            elif w.distortion == "alie":
+                if w.copy_noise:
+                    z = normal_np(w.seed, STREAM_COPY0 + 8 * i + s, c0, c1)
+                    out[i, s, : c1 - c0] = (g.astype(np.float64) + w.copy_noise * z).astype(np.float32)
+                else:
+                    out[i, s, : c1 - c0] = g
+            elif w.distortion in ("alie", "foe"):
                 out[i, s, : c1 - c0] = bad
             else:
                 out[i, s, : c1 - c0] = (g.astype(np.float64) * -w.scale).astype(np.float32)
@@ -313,15 +328,19 @@ def build_copies_torch(w: Workload, file_workers: np.ndarray, device, out=None,
         out[:, :, d:] = pad_value
     mask = corrupted_mask(w, fw)
     bad = None
-    if mask.any() and w.distortion == "alie":
+    if mask.any() and w.distortion in ("alie", "foe"):
         bad = _alie_torch(w, 0, d, device)
     b = 0.01 * normal_torch(w.seed, STREAM_B, 0, d, device)
     for i in range(f):
         g = honest_torch(w.seed, i, 0, d, device, b)
         for s in range(r):
             if not mask[i, s]:
-                out[i, s, :d].copy_(g)
-            elif w.distortion == "alie":
+                if w.copy_noise:
+                    z = normal_torch(w.seed, STREAM_COPY0 + 8 * i + s, 0, d, device)
+                    out[i, s, :d].copy_((g.to(torch.float64) + w.copy_noise * z).to(torch.float32))
+                else:
+                    out[i, s, :d].copy_(g)
+            elif w.distortion in ("alie", "foe"):
                 out[i, s, :d].copy_(bad)
             else:
                 out[i, s, :d].copy_((g.to(torch.float64) * -w.scale).to(torch.float32))
