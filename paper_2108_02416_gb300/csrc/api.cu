@@ -31,7 +31,40 @@ using namespace aspis;
 
 namespace {
 
-// Host-to-device copies of the round's inputs are split over kLanes streams
+// Pinned host memory is mapped into the device's address space, and over the
+// Grace-Blackwell host link SM loads of it stream at the link's rate (about
+// 205 GB/s for a 61 GB buffer, steady from run to run) where the copy engines
+// moved the same buffer at 135-210 GB/s.  So a large copy from a
+// device-mapped host buffer is a grid-stride kernel of 16-byte loads and
+// stores; returns false (nothing enqueued) when the buffer is not
+// device-mapped or not 16-byte aligned, and the copy engines take it.
+__global__ void __launch_bounds__(256)
+h2d_copy_kernel(const uint4 *__restrict__ src, uint4 *__restrict__ dst, int64_t n16)
+{
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16;
+         i += (int64_t)gridDim.x * blockDim.x)
+        dst[i] = __ldcs(src + i);
+}
+
+bool h2d_sm(void *dst, const void *src, size_t bytes, cudaStream_t st, cudaError_t &err)
+{
+    cudaPointerAttributes at{};
+    if (cudaPointerGetAttributes(&at, src) != cudaSuccess) {
+        cudaGetLastError();                          // not a pointer CUDA knows: clear the error
+        return false;
+    }
+    if (at.type != cudaMemoryTypeHost || !at.devicePointer) return false;
+    if (((uintptr_t)at.devicePointer | (uintptr_t)dst | (uintptr_t)bytes) % 16 != 0) return false;
+    const int64_t n16 = (int64_t)(bytes / 16);
+    int64_t grid = (int64_t)sm_count() * 8;
+    if (grid > (n16 + 255) / 256) grid = (n16 + 255) / 256;
+    h2d_copy_kernel<<<(unsigned)grid, 256, 0, st>>>(static_cast<const uint4 *>(at.devicePointer),
+                                                    static_cast<uint4 *>(dst), n16);
+    err = cudaGetLastError();
+    return true;
+}
+
+// Other host-to-device copies of the round's inputs are split over kLanes streams
 // so that several copy engines move them at once; the caller's stream waits
 // for all of them.  Streams and events are created once per device.
 constexpr int kLanes = 4;
@@ -215,7 +248,10 @@ extern "C" aspis_status aspis_round_host(const float *host_copies, float *dev_co
     if ((s = check_copies(dev_copies, d, ld, a)) != ASPIS_OK) return s;
     cudaStream_t st = (cudaStream_t)stream;
     const size_t bytes = sizeof(float) * (size_t)(a->f * a->r) * (size_t)ld;
-    if (h2d_split(dev_copies, host_copies, bytes, st) != cudaSuccess) return ASPIS_E_CUDA;
+    cudaError_t e = cudaSuccess;
+    const bool by_sm = bytes >= ((size_t)64 << 20) && h2d_sm(dev_copies, host_copies, bytes, st, e);
+    if (!by_sm) e = h2d_split(dev_copies, host_copies, bytes, st);
+    if (e != cudaSuccess) return ASPIS_E_CUDA;
     s = aspis_round(dev_copies, d, ld, a, file_neq, adj, det, sel, mode, dev_out, stream);
     if (s != ASPIS_OK) return s;
     if (cudaMemcpyAsync(host_out, dev_out, sizeof(float) * (size_t)d, cudaMemcpyDeviceToHost,

@@ -310,6 +310,35 @@ def test_round_host_entry_point():
     assert det.success == want.det.success and det.n_sel == want.n_sel
 
 
+@pytest.mark.parametrize("kind", ["pinned", "pinned_offset", "pageable"])
+def test_round_host_large_copy_paths(kind):
+    """Above 64 MiB the host copy takes the copy kernel (pinned, aligned) or
+    the copy engines (pinned at an odd offset, pageable); results are the
+    oracle's either way."""
+    import dataclasses
+    w = dataclasses.replace(synth.CONFIGS["k15_r3_d11m_strong_alie"], d=20000)   # 109 MB
+    oa = oracle.assign(w.K, w.r)
+    arr = synth.build_copies_np(w, oa.file_workers)
+    want = oracle.run_round(arr, oa, w.d)
+    if kind == "pageable":
+        host = torch.from_numpy(arr)
+    else:
+        base = torch.empty(arr.size + 1, dtype=torch.float32).pin_memory()
+        off = 1 if kind == "pinned_offset" else 0
+        host = base[off: off + arr.size].view(arr.shape)
+        host.copy_(torch.from_numpy(arr))
+    a = ap.aspis_assign(w.K, w.r)
+    buf = ap.RoundBuffers(a, w.d, DEV)
+    dev = torch.empty(arr.shape, dtype=torch.float32, device=DEV)
+    hout = torch.empty(w.d, dtype=torch.float32).pin_memory()
+    hdet = torch.zeros(ap.DETECTION_BYTES, dtype=torch.uint8).pin_memory()
+    ap.aspis_round_host(host, dev, w.d, a, buf.file_neq, buf.adj, buf.det, buf.sel, buf.out,
+                        hout, hdet)
+    torch.cuda.synchronize()
+    assert torch.equal(dev.cpu().view(torch.int32), torch.from_numpy(arr).view(torch.int32))
+    assert np.array_equal(hout.numpy().view(np.uint32), want.out.view(np.uint32))
+
+
 def test_generator_torch_cuda_matches_numpy():
     """The shared input generator gives the same bits on the GPU and the CPU."""
     w = synth.Workload("g", K=7, r=3, d=1000, q=2, attack="strong", seed=5)
