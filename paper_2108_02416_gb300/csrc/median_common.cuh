@@ -11,7 +11,6 @@ constexpr int kNB = 128;          // histogram rows (value-space bins use 0..126
 constexpr int kLogNB = 7;
 constexpr int kTopBin = 126;      // value-space bins are 0..kTopBin
 constexpr uint32_t kPadTag = 0x7Fu;   // tag byte of a missing row: no value-space bin
-constexpr int kCap = 32;          // keys ranked directly
 
 // IEEE totalOrder as unsigned order: flip all bits of negatives, the sign
 // bit of non-negatives.  A bijection, so the median's bits come back exactly.
