@@ -225,11 +225,12 @@ aspis_status aspis_round_static(const float *copies, int64_t d, int64_t ld,
  * dev_copies, runs aspis_round, and copies the d aggregated floats into
  * host_out and the detection record into host_det.  All work and copies are
  * ordered on the stream.  Copies of 64 MiB or more from pinned host memory
- * that the device can address (16-byte aligned) are made by a copy kernel
- * whose SM loads stream over the host link; other copies of 64 MiB or more
- * are split over four library-owned streams, created on first use, that the
- * stream waits for.  The host buffers must stay valid until the stream is
- * synchronized.  Device
+ * that the device can address (16-byte aligned, ld % 4 == 0) are made by a
+ * copy kernel whose SM loads stream over the host link, in eight file-aligned
+ * chunks, and each chunk is compared on a library-owned stream (created on
+ * first use) as soon as it has landed; other copies of 64 MiB or more are
+ * split over four library-owned streams that the stream waits for.  The host
+ * buffers must stay valid until the stream is synchronized.  Device
  * buffers are the caller's, as for aspis_round. */
 aspis_status aspis_round_host(const float *host_copies, float *dev_copies,
                               int64_t d, int64_t ld, const aspis_assignment *a,

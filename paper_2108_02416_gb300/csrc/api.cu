@@ -64,6 +64,74 @@ bool h2d_sm(void *dst, const void *src, size_t bytes, cudaStream_t st, cudaError
     return true;
 }
 
+// The copy and the compare of aspis_round_host overlap for pinned inputs: the
+// copy kernel moves file-aligned chunks over the host link on the caller's
+// stream with two CTAs per SM (the link saturates well below that), and each
+// chunk's compare runs on a library-owned stream as soon as the chunk has
+// landed, on the SMs the copy leaves free.  Only the last chunk's compare,
+// the graph and the rest of the round follow the last byte.  Events are
+// recorded and waited on under one lock, so concurrent callers cannot mix
+// them up (their compares then share the side stream).
+constexpr int kPipeChunks = 8;
+struct PipeLanes {
+    bool ready = false;
+    cudaStream_t side;
+    cudaEvent_t landed[kPipeChunks], compared;
+};
+std::mutex g_pipe_mu;
+PipeLanes g_pipe[64];
+
+bool copy_and_compare(const float *host, float *dev, int64_t d, int64_t ld,
+                      const aspis_assignment *a, uint32_t *file_neq, cudaStream_t st,
+                      cudaError_t &err)
+{
+    cudaPointerAttributes at{};
+    if (cudaPointerGetAttributes(&at, host) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    if (at.type != cudaMemoryTypeHost || !at.devicePointer) return false;
+    // every chunk starts at a file boundary: 16-byte aligned when ld % 4 == 0
+    if (((uintptr_t)at.devicePointer | (uintptr_t)dev) % 16 != 0 || ld % 4 != 0) return false;
+    int devno = 0;
+    if ((err = cudaGetDevice(&devno)) != cudaSuccess) return true;
+    if (devno < 0 || devno >= 64) return false;
+    std::lock_guard<std::mutex> g(g_pipe_mu);
+    PipeLanes &L = g_pipe[devno];
+    if (!L.ready) {
+        if ((err = cudaStreamCreateWithFlags(&L.side, cudaStreamNonBlocking)) != cudaSuccess) return true;
+        for (int k = 0; k < kPipeChunks; ++k)
+            if ((err = cudaEventCreateWithFlags(&L.landed[k], cudaEventDisableTiming)) != cudaSuccess)
+                return true;
+        if ((err = cudaEventCreateWithFlags(&L.compared, cudaEventDisableTiming)) != cudaSuccess)
+            return true;
+        L.ready = true;
+    }
+    const int64_t f = a->f, r = a->r, row = r * ld;               // floats per file
+    if ((err = cudaMemsetAsync(file_neq, 0, sizeof(uint32_t) * (size_t)f, st)) != cudaSuccess)
+        return true;
+    const int64_t per = (f + kPipeChunks - 1) / kPipeChunks;
+    const float *src = static_cast<const float *>(at.devicePointer);
+    for (int k = 0; k < kPipeChunks; ++k) {
+        const int64_t i0 = k * per, i1 = i0 + per < f ? i0 + per : f;
+        if (i0 >= i1) break;
+        const int64_t n16 = (i1 - i0) * row / 4;
+        int64_t grid = (int64_t)sm_count() * 2;
+        if (grid > (n16 + 255) / 256) grid = (n16 + 255) / 256;
+        h2d_copy_kernel<<<(unsigned)grid, 256, 0, st>>>(reinterpret_cast<const uint4 *>(src + i0 * row),
+                                                        reinterpret_cast<uint4 *>(dev + i0 * row), n16);
+        if ((err = cudaGetLastError()) != cudaSuccess) return true;
+        if ((err = cudaEventRecord(L.landed[k], st)) != cudaSuccess) return true;
+        if ((err = cudaStreamWaitEvent(L.side, L.landed[k], 0)) != cudaSuccess) return true;
+        if ((err = launch_compare(dev + i0 * row, i1 - i0, (int)r, d, ld, file_neq + i0, L.side)) !=
+            cudaSuccess)
+            return true;
+    }
+    if ((err = cudaEventRecord(L.compared, L.side)) != cudaSuccess) return true;
+    err = cudaStreamWaitEvent(st, L.compared, 0);
+    return true;
+}
+
 // Other host-to-device copies of the round's inputs are split over kLanes streams
 // so that several copy engines move them at once; the caller's stream waits
 // for all of them.  Streams and events are created once per device.
@@ -248,12 +316,28 @@ extern "C" aspis_status aspis_round_host(const float *host_copies, float *dev_co
     if ((s = check_copies(dev_copies, d, ld, a)) != ASPIS_OK) return s;
     cudaStream_t st = (cudaStream_t)stream;
     const size_t bytes = sizeof(float) * (size_t)(a->f * a->r) * (size_t)ld;
+    if (!file_neq || !adj || !det || !sel || !dev_out || (mode != 0 && mode != 1))
+        return ASPIS_E_INVAL;
+    if (a->f > ASPIS_MAX_AGG_FILES) return ASPIS_E_RANGE;
     cudaError_t e = cudaSuccess;
-    const bool by_sm = bytes >= ((size_t)64 << 20) && h2d_sm(dev_copies, host_copies, bytes, st, e);
-    if (!by_sm) e = h2d_split(dev_copies, host_copies, bytes, st);
+    const bool piped = bytes >= ((size_t)64 << 20) &&
+                       copy_and_compare(host_copies, dev_copies, d, ld, a, file_neq, st, e);
     if (e != cudaSuccess) return ASPIS_E_CUDA;
-    s = aspis_round(dev_copies, d, ld, a, file_neq, adj, det, sel, mode, dev_out, stream);
-    if (s != ASPIS_OK) return s;
+    if (piped) {
+        // the copies are on the device and compared: the rest of the round
+        if ((s = aspis_graph(file_neq, a, adj, stream)) != ASPIS_OK) return s;
+        if ((s = aspis_detect(adj, a->K, det, stream)) != ASPIS_OK) return s;
+        if ((s = aspis_select(file_neq, det, a, sel, stream)) != ASPIS_OK) return s;
+        if ((s = aspis_aggregate(dev_copies, d, ld, a, sel, det, mode, dev_out, stream)) != ASPIS_OK)
+            return s;
+    } else {
+        const bool by_sm =
+            bytes >= ((size_t)64 << 20) && h2d_sm(dev_copies, host_copies, bytes, st, e);
+        if (!by_sm) e = h2d_split(dev_copies, host_copies, bytes, st);
+        if (e != cudaSuccess) return ASPIS_E_CUDA;
+        s = aspis_round(dev_copies, d, ld, a, file_neq, adj, det, sel, mode, dev_out, stream);
+        if (s != ASPIS_OK) return s;
+    }
     if (cudaMemcpyAsync(host_out, dev_out, sizeof(float) * (size_t)d, cudaMemcpyDeviceToHost,
                         st) != cudaSuccess)
         return ASPIS_E_CUDA;
