@@ -3,7 +3,7 @@ against the oracle: mismatch words, graph, clique, slot masks, the kept
 files' averages and the median, bit for bit; the mean within its tolerance.
 Cases: tau = 0 on bit-identical copies (equal to the exact round), honest
 copies with per-copy noise below tau under the weak, optimal and
-all-adversary attacks (Case 1 averages, Case 2 clusters, r = 3 and 5), the
+all-adversary attacks (Case 1 averages, Case 2 clusters, r = 2 to 6), the
 Fall-of-Empires distortion, NaNs, the 4-byte paths, and the full ResNet-18
 length."""
 import dataclasses
@@ -94,6 +94,17 @@ def test_tolerant_unaligned_paths(offset, ldm_pad):
     host = synth.build_copies_np(w, oa.file_workers)
     want = oracle.run_round_tolerant(host, oa, 1e-4, w.d, 0)
     check(run(host, w, 1e-4, 0, offset, ldm_pad), want, 0)
+
+
+@pytest.mark.parametrize("K,r,q,attack", [(6, 2, 2, "weak"), (8, 2, 3, "strong"), (8, 4, 3, "strong"),
+                                          (9, 4, 4, "weak"), (9, 6, 4, "strong")])
+def test_tolerant_other_r(K, r, q, attack):
+    w = synth.Workload("tol_r", K=K, r=r, d=1003, q=q, attack=attack, distortion="alie", seed=K + r,
+                       copy_noise=1e-6)
+    oa = oracle.assign(w.K, w.r)
+    host = synth.build_copies_np(w, oa.file_workers)
+    want = oracle.run_round_tolerant(host, oa, 1e-4, w.d, 0)
+    check(run(host, w, 1e-4), want)
 
 
 def test_tolerant_foe_and_nans():
