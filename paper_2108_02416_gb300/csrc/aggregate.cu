@@ -94,6 +94,11 @@ __device__ __forceinline__ void cp_async4(uint32_t saddr, const void *g)
     asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(saddr), "l"(g) : "memory");
 }
 
+__device__ __forceinline__ void prefetch_l2(const void *p)
+{
+    asm volatile("prefetch.global.L2 [%0];\n" ::"l"(p));
+}
+
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
@@ -133,8 +138,12 @@ __device__ __forceinline__ uint32_t pack4(uint32_t b0, uint32_t b1, uint32_t b2,
 template <int V>
 struct Geo {
     static constexpr int TC = 32 * V;                 // coordinates per tile
-    static constexpr int NP = V >= 2 ? V / 2 : 1;     // histogram words per (bin, lane)
-    static constexpr int SHB = NP == 2 ? 8 : 7;       // log2 of the bytes per histogram row
+    static constexpr int NP = V >= 2 ? V / 2 : 1;     // key-space histogram words per (bin, lane)
+    static constexpr int SHB = NP == 2 ? 8 : 7;       // log2 of the bytes per key-space row
+    // value-space histogram: one word per (bin, lane) holding the lane's V
+    // counters, 8-bit for V = 4 (an overflow is detected by the bin search),
+    // 16-bit otherwise
+    static constexpr int HW = kVB * 32 > kNB * NP * 32 ? kVB * 32 : kNB * NP * 32;   // histogram words
     static constexpr int RPW = 4 / V;                 // rows per tag word
     static constexpr int CAP = kListWords / TC;       // list entries per coordinate
 };
@@ -143,7 +152,7 @@ struct Layout {
     size_t tags, hist, list, state, rows, total;
 };
 
-template <int V, int NT>
+template <int V, int NT, int MODE>
 __host__ __device__ inline Layout make_layout(int64_t f)
 {
     using G = Geo<V>;
@@ -152,8 +161,8 @@ __host__ __device__ inline Layout make_layout(int64_t f)
     const int64_t per_slot = (f + kWarps - 1) / kWarps;
     const int64_t jw = (per_slot + G::RPW - 1) / G::RPW;     // tag words per thread
     size_t o = 0;
-    L.tags = o; o += (size_t)jw * kWarps * 32 * 4;
-    L.hist = o; o += (size_t)kNB * G::NP * 32 * 4;
+    L.tags = o; o += MODE == 0 ? (size_t)jw * kWarps * 32 * 4 : 0;     // the mean keeps no tags
+    L.hist = o; o += (size_t)G::HW * 4;
     L.list = o; o += (size_t)kListWords * 4;         // also the bin-search and mean partials
     L.state = o; o += (size_t)kStateWords * G::TC * 4;
     L.rows = o; o += ((size_t)f * 2 + 15) / 16 * 16;
@@ -170,14 +179,15 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     using T = typename Vec<V>::T;
     constexpr int TC = G::TC, NP = G::NP, SHB = G::SHB, RPW = G::RPW, CAP = G::CAP;
     constexpr int kThreads = NT, kWarps = NT / 32;           // warps = row slots of a CTA
-    constexpr int kBPW = (kNB + kWarps - 1) / kWarps;        // bins per warp in the bin search
+    constexpr int kBPW = (kVB + kWarps - 1) / kWarps;        // bins per warp in the bin search
+    constexpr int HW = G::HW;
     // rows per load batch and thread: deeper for narrow rows when one CTA
     // has the SM's registers
     constexpr int kU = (MINB >= 2 || V == 4) ? 8 : 24;
     extern __shared__ __align__(16) unsigned char smem[];
-    const Layout L = make_layout<V, NT>(f);
+    const Layout L = make_layout<V, NT, MODE>(f);
     uint32_t *tags = reinterpret_cast<uint32_t *>(smem + L.tags);     // [word][kWarps][32]
-    uint32_t *hist = reinterpret_cast<uint32_t *>(smem + L.hist);     // [kNB][NP][32]
+    uint32_t *hist = reinterpret_cast<uint32_t *>(smem + L.hist);     // [kVB][32] or [kNB][NP][32]
     uint32_t *list = reinterpret_cast<uint32_t *>(smem + L.list);     // [CAP][TC]
     uint32_t *st = reinterpret_cast<uint32_t *>(smem + L.state);      // [kStateWords][TC]
     uint16_t *rows = reinterpret_cast<uint16_t *>(smem + L.rows);
@@ -211,6 +221,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
         return;
     }
     const uint32_t krank = (uint32_t)((n - 1) / 2);
+    const bool widen = V == 4 && n > 512;
     const int nmine = n > w ? (n - w + kWarps - 1) / kWarps : 0;     // rows of this warp
     const int nwords = (nmine + RPW - 1) / RPW;
     const int64_t ntiles = (d + TC - 1) / TC;
@@ -223,7 +234,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
         S(S_LCNT, i) = 0u;
         S(S_PCNT, i) = 0u;
     }
-    for (int i = tid * 4; i < kNB * NP * 32; i += kThreads * 4)
+    for (int i = tid * 4; i < HW; i += kThreads * 4)
         *reinterpret_cast<uint4 *>(hist + i) = make_uint4(0u, 0u, 0u, 0u);
 
     // address of row j of this warp at the lane's chunk of a tile
@@ -345,6 +356,11 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                         fn(xa[u], j0 + u, u);
                         const int jn = j0 + kU + u;
                         if (lv && jn < nmine) xa[u] = load_row<V>(row_ptr(lb, jn));
+                        if constexpr (V == 4) {
+                            // the row of the batch after next into L2: the four
+                            // 128-byte lines of a row segment, one per 8 lanes
+                            if (lv && jn + kU < nmine && (lane & 7) == 0) prefetch_l2(row_ptr(lb, jn + kU));
+                        }
                     }
                 }
             };
@@ -410,14 +426,18 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             }
             __syncthreads();                                        // (B)
             float vs[V], vc[V];
-            uint32_t hb[NP];
 #pragma unroll
             for (int k = 0; k < V; ++k) {
                 const float xlo = __uint_as_float(from_key(S(S_MIN, lane * V + k)));
                 const float xhi = __uint_as_float(from_key(S(S_MAX, lane * V + k)));
-                // sample range -> y in [1/126, 125/126]: bins 1..125
-                const float sc = (124.0f / 126.0f) / (xhi - xlo);
-                const float cc = fmaf(-xlo, sc, 1.0f / 126.0f);
+                // sample range -> y in [1/254, 253/254]: bins 1..253.  With
+                // 8-bit counters and more than 512 kept files, the bins span
+                // twice the sample range, so that the two outer bins (the
+                // values outside it) stay far below 256 members
+                const float wd = widen ? 2.0f * (xhi - xlo) : xhi - xlo;
+                const float x0 = widen ? xlo - 0.5f * (xhi - xlo) : xlo;
+                const float sc = (252.0f / 254.0f) / wd;
+                const float cc = fmaf(-x0, sc, 1.0f / 254.0f);
                 const bool ok = isfinite(xlo) && isfinite(xhi) && xhi > xlo && isfinite(sc) &&
                                 sc > 0.f && isfinite(cc);
                 vs[k] = ok ? sc : 0.f;
@@ -427,9 +447,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     S(S_MODE, lane * V + k) = !live ? M_DONE : (ok ? M_VH : M_KA);
                 }
             }
-#pragma unroll
-            for (int p = 0; p < NP; ++p)
-                hb[p] = hist_s + (uint32_t)(p * 32 + lane) * 4u - (0x4B000000u << SHB);
+            const uint32_t hb = hist_s + (uint32_t)lane * 4u - (0x4B000000u << 7);
 
             // ---- sweep: the pending tile's members (old tag words), then
             // VH for this tile (histogram, new tag words, NaN check)
@@ -439,9 +457,16 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
 #pragma unroll
                 for (int k = 0; k < V; ++k) {
                     bb[k] = vbin_bits(__uint_as_float(elem<V>(x, k)), vs[k], vc[k]);
-                    const uint32_t a = (bb[k] << SHB) + hb[k / 2];
-                    if (k & 1) red_shared<0x10000u>(a);
-                    else red_shared<1u>(a);
+                    const uint32_t a = (bb[k] << 7) + hb;
+                    if constexpr (V == 4) {
+                        if (k == 0) red_shared<1u>(a);
+                        else if (k == 1) red_shared<0x100u>(a);
+                        else if (k == 2) red_shared<0x10000u>(a);
+                        else red_shared<0x1000000u>(a);
+                    } else {
+                        if (k & 1) red_shared<0x10000u>(a);
+                        else red_shared<1u>(a);
+                    }
                 }
                 if constexpr (V == 4) {
                     nan_check(nanf, __uint_as_float(x.x), __uint_as_float(x.y),
@@ -486,26 +511,35 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             __syncthreads();                                        // (R)
             for (int c = tid; c < TC; c += kThreads) S(S_LCNT, c) = 0u;
 
-            // ---- B1: per-warp partial sums over bins [kBPW*w, kBPW*w + kBPW)
+            // ---- B1: per-warp partial sums over bins [kBPW*w, kBPW*w + kBPW);
+            // 8-bit counters are summed as two pairs of 16-bit fields
             {
-                uint32_t ps[NP];
-#pragma unroll
-                for (int p = 0; p < NP; ++p) ps[p] = 0u;
+                uint32_t ps0 = 0u, ps1 = 0u;
 #pragma unroll
                 for (int b = 0; b < kBPW; ++b)
-                    if (w * kBPW + b < kNB)
+                    if (w * kBPW + b < kVB) {
+                        const uint32_t x = hist[(w * kBPW + b) * 32 + lane];
+                        if constexpr (V == 4) {
+                            ps0 += x & 0x00FF00FFu;
+                            ps1 += (x >> 8) & 0x00FF00FFu;
+                        } else {
+                            ps0 += x;
+                        }
+                    }
 #pragma unroll
-                        for (int p = 0; p < NP; ++p) ps[p] += hist[((w * kBPW + b) * NP + p) * 32 + lane];
-#pragma unroll
-                for (int k = 0; k < V; ++k)
-                    list[w * TC + lane * V + k] = (ps[k / 2] >> (16 * (k & 1))) & 0xFFFFu;
+                for (int k = 0; k < V; ++k) {
+                    uint32_t pk;
+                    if constexpr (V == 4) pk = (((k & 1) ? ps1 : ps0) >> (16 * (k >> 1))) & 0xFFFFu;
+                    else pk = (ps0 >> (16 * (k & 1))) & 0xFFFFu;
+                    list[w * TC + lane * V + k] = pk;
+                }
             }
             __syncthreads();                                        // (D)
             // ---- B2: one thread per coordinate resolves its bin
             for (int c = tid; c < TC; c += kThreads) {
                 uint32_t pc = 0u;
                 if (S(S_MODE, c) == M_VH) {
-                    uint32_t rem = krank;
+                    uint32_t rem = krank, tot = 0u;
                     int owner = kWarps - 1;
                     bool fd = false;
                     for (int u = 0; u < kWarps; ++u) {
@@ -514,15 +548,17 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                         if (hit) owner = u;
                         if (!fd && !hit) rem -= pu;
                         fd |= hit;
+                        tot += pu;
                     }
                     const int lc = c / V, k = c % V;
-                    const uint32_t *h = hist + (k / 2) * 32 + lc;
-                    const int shf = 16 * (k & 1);
-                    int bin = min(owner * kBPW + kBPW, kNB) - 1;
+                    const uint32_t *h = hist + lc;
+                    const int shf = V == 4 ? 8 * k : 16 * (k & 1);
+                    const uint32_t msk = V == 4 ? 0xFFu : 0xFFFFu;
+                    int bin = min(owner * kBPW + kBPW, kVB) - 1;
                     uint32_t cnt = 0u;
                     bool f2 = false;
-                    for (int b = owner * kBPW; b < min(owner * kBPW + kBPW, kNB); ++b) {
-                        const uint32_t cb = (h[b * NP * 32] >> shf) & 0xFFFFu;
+                    for (int b = owner * kBPW; b < min(owner * kBPW + kBPW, kVB); ++b) {
+                        const uint32_t cb = (h[b * 32] >> shf) & msk;
                         const bool hit = !f2 && rem < cb;
                         if (hit) {
                             bin = b;
@@ -535,14 +571,16 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     S(S_REM, c) = rem;
                     S(S_CNT, c) = cnt;
                     S(S_PREM, c) = rem;
-                    const bool vcm = cnt <= (uint32_t)CAP;
-                    S(S_MODE, c) = vcm ? M_VC : M_VM;
+                    // an 8-bit counter that overflowed changes its coordinate's total
+                    const bool exact = tot == (uint32_t)n;
+                    const bool vcm = exact && cnt <= (uint32_t)CAP;
+                    S(S_MODE, c) = !exact ? M_KA : (vcm ? M_VC : M_VM);
                     pc = vcm ? cnt : 0u;
                 }
                 S(S_PCNT, c) = pc;
             }
             __syncthreads();                                        // (E)
-            for (int i = tid * 4; i < kNB * NP * 32; i += kThreads * 4)
+            for (int i = tid * 4; i < HW; i += kThreads * 4)
                 *reinterpret_cast<uint4 *>(hist + i) = make_uint4(0u, 0u, 0u, 0u);
 
             // this tile becomes the pending one: target bins of its coordinates
@@ -681,7 +719,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                         S(S_LCNT, c) = 0u;
                     }
                     __syncthreads();
-                    for (int i = tid * 4; i < kNB * NP * 32; i += kThreads * 4)
+                    for (int i = tid * 4; i < HW; i += kThreads * 4)
                         *reinterpret_cast<uint4 *>(hist + i) = make_uint4(0u, 0u, 0u, 0u);
                     bool more = false;
                     for (int c = tid; c < TC; c += kThreads) {
@@ -703,6 +741,126 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     }
 }
 
+// Lower median for more kept files than the tag bytes of even a 32-coordinate
+// tile can hold in shared memory (about 5,800): an exact 8-bit radix select
+// on the totalOrder keys, four passes per tile, each re-reading the tile's
+// kept values.  A tile is 32 coordinates (lane l of every warp holds
+// coordinate l; the warps split the rows); the histogram has one 32-bit
+// counter per (digit, coordinate).  Four times the reads of the tagged
+// kernel, no per-value state.
+constexpr int kRadixThreads = 256;
+
+__global__ void __launch_bounds__(kRadixThreads)
+median_radix_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, int64_t ld,
+                    const int8_t *__restrict__ sel, aspis_detection *det, float *__restrict__ out)
+{
+    constexpr int kW = kRadixThreads / 32;
+    extern __shared__ __align__(16) unsigned char smem[];
+    uint32_t *hist = reinterpret_cast<uint32_t *>(smem);              // [256 digits][32 coordinates]
+    uint32_t *pre = hist + 256 * 32;                                  // per coordinate: key prefix
+    uint32_t *rnk = pre + 32;                                         // per coordinate: rank left
+    uint16_t *rows = reinterpret_cast<uint16_t *>(rnk + 32);         // kept rows
+    __shared__ int warp_tot[kW];
+    const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+    const unsigned full = 0xffffffffu;
+    int n = 0;
+    for (int64_t b0 = 0; b0 < f; b0 += kRadixThreads) {
+        const int64_t i = b0 + tid;
+        const int sv = i < f ? (int)sel[i] : -1;
+        const unsigned m = __ballot_sync(full, sv >= 0);
+        if (lane == 0) warp_tot[w] = __popc(m);
+        __syncthreads();
+        int off = n, tot = 0;
+        for (int u = 0; u < kW; ++u) {
+            off += u < w ? warp_tot[u] : 0;
+            tot += warp_tot[u];
+        }
+        if (sv >= 0) rows[off + __popc(m & ((1u << lane) - 1u))] = (uint16_t)(i * r + sv);
+        n += tot;
+        __syncthreads();
+    }
+    if (n == 0) {
+        if (blockIdx.x == 0 && tid == 0) det->status = ASPIS_E_EMPTY;
+        return;
+    }
+    const uint32_t krank = (uint32_t)((n - 1) / 2);
+    const int64_t ntiles = (d + 31) / 32;
+    for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x) {
+        const int64_t col = t * 32 + lane;
+        const bool live = col < d;
+        if (tid < 32) {
+            pre[tid] = 0u;
+            rnk[tid] = krank;
+        }
+        for (int p = 0; p < 4; ++p) {
+            const int sh = 24 - 8 * p;
+            const uint32_t pmask = p == 0 ? 0u : 0xFFFFFFFFu << (32 - 8 * p);
+            for (int i = tid; i < 256 * 32; i += kRadixThreads) hist[i] = 0u;
+            __syncthreads();
+            const uint32_t want = pre[lane];
+            for (int j0 = w; j0 < n; j0 += kW * 8) {
+                uint32_t v[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int j = j0 + u * kW;
+                    v[u] = live && j < n ? __ldcg(reinterpret_cast<const unsigned int *>(
+                                               copies + (int64_t)rows[j] * ld + col))
+                                         : 0u;
+                }
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int j = j0 + u * kW;
+                    const uint32_t key = to_key(v[u]);
+                    if (live && j < n && (key & pmask) == want)
+                        atomicAdd(&hist[((key >> sh) & 0xFFu) * 32 + lane], 1u);
+                }
+            }
+            __syncthreads();
+            // warp w settles coordinates 4w..4w+3: a warp scan over the 256 digits
+            for (int q = 0; q < 4; ++q) {
+                const int cc = 4 * w + q;
+                uint32_t cb[8], sum = 0u;
+#pragma unroll
+                for (int b = 0; b < 8; ++b) {
+                    cb[b] = hist[(lane * 8 + b) * 32 + cc];
+                    sum += cb[b];
+                }
+                uint32_t inc = sum;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const uint32_t y = __shfl_up_sync(full, inc, o);
+                    if (lane >= o) inc += y;
+                }
+                const uint32_t rk = rnk[cc], exc = inc - sum;
+                const bool mine = exc <= rk && rk < inc;
+                uint32_t dig = 0u, r2 = rk - exc;
+                if (mine) {
+                    bool hit = false;
+#pragma unroll
+                    for (int b = 0; b < 8; ++b) {
+                        if (!hit && r2 < cb[b]) {
+                            dig = (uint32_t)(lane * 8 + b);
+                            hit = true;
+                        }
+                        if (!hit) r2 -= cb[b];
+                    }
+                }
+                const unsigned bal = __ballot_sync(full, mine);
+                const int src = bal ? __ffs(bal) - 1 : 0;
+                dig = __shfl_sync(full, dig, src);
+                r2 = __shfl_sync(full, r2, src);
+                if (lane == 0 && bal) {
+                    pre[cc] |= dig << sh;
+                    rnk[cc] = r2;
+                }
+            }
+            __syncthreads();
+        }
+        if (w == 0 && live) out[col] = __uint_as_float(from_key(pre[lane]));
+        __syncthreads();
+    }
+}
+
 size_t smem_cap()
 {
     int dev = 0, cap = 0;
@@ -717,7 +875,7 @@ cudaError_t try_launch(bool &launched, const float *copies, int64_t f, int r, in
                        cudaStream_t stream)
 {
     launched = false;
-    const Layout L = make_layout<V, NT>(f);
+    const Layout L = make_layout<V, NT, MODE>(f);
     if (L.total > smem_cap()) return cudaSuccess;
     auto kern = aggregate_kernel<V, MINB, W32, MODE, NT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -732,6 +890,24 @@ cudaError_t try_launch(bool &launched, const float *copies, int64_t f, int r, in
     if (grid > ntiles) grid = ntiles;
     kern<<<(unsigned)grid, NT, L.total, stream>>>(copies, f, r, d, ld, sel, det, out);
     launched = true;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_radix(const float *copies, int64_t f, int r, int64_t d, int64_t ld,
+                         const int8_t *sel, aspis_detection *det, float *out, cudaStream_t stream)
+{
+    const size_t smem = (size_t)(256 * 32 + 64) * 4 + ((size_t)f * 2 + 15) / 16 * 16;
+    if (smem > smem_cap()) return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(median_radix_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, median_radix_kernel, kRadixThreads, smem);
+    if (e != cudaSuccess) return e;
+    const int64_t ntiles = (d + 31) / 32;
+    int64_t grid = (int64_t)sm_count() * (per_sm > 0 ? per_sm : 1);
+    if (grid > ntiles) grid = ntiles;
+    median_radix_kernel<<<(unsigned)grid, kRadixThreads, smem, stream>>>(copies, f, r, d, ld, sel, det, out);
     return cudaGetLastError();
 }
 
@@ -759,6 +935,7 @@ cudaError_t launch_mode(int align, const float *copies, int64_t f, int r, int64_
     ASPIS_TRY(1, 2, 384)
     ASPIS_TRY(1, 1, 384)
 #undef ASPIS_TRY
+    if constexpr (MODE == 0) return launch_radix(copies, f, r, d, ld, sel, det, out, stream);
     return cudaErrorInvalidValue;
 }
 

@@ -7,10 +7,11 @@
 
 namespace aspis {
 
-constexpr int kNB = 128;          // histogram rows (value-space bins use 0..126)
-constexpr int kLogNB = 7;
-constexpr int kTopBin = 126;      // value-space bins are 0..kTopBin
-constexpr uint32_t kPadTag = 0x7Fu;   // tag byte of a missing row: no value-space bin
+constexpr int kNB = 128;          // key-space histogram rows of the exact path
+constexpr int kLogNB = 7;         // key bits resolved per key-space pass
+constexpr int kVB = 256;          // value-space histogram rows
+constexpr int kTopBin = 254;      // value-space bins are 0..kTopBin
+constexpr uint32_t kPadTag = 0xFFu;   // tag byte of a missing row: no value-space bin
 
 // IEEE totalOrder as unsigned order: flip all bits of negatives, the sign
 // bit of non-negatives.  A bijection, so the median's bits come back exactly.
@@ -25,8 +26,8 @@ __device__ __forceinline__ uint32_t from_key(uint32_t k)
 }
 
 // Value-space bin of x, as the bits of 2^23 + bin: y = sat(x*s + c) in
-// [0, 1] (fma with saturation: NaN gives +0), then 2^23 + rint(126*y), whose
-// low byte is the bin 0..126.  Both steps are correctly rounded and
+// [0, 1] (fma with saturation: NaN gives +0), then 2^23 + rint(254*y), whose
+// low byte is the bin 0..254.  Both steps are correctly rounded and
 // non-decreasing, so the map is monotone in the IEEE totalOrder of every
 // non-NaN x (+0 and -0 share a bin) and always lands in 0..126, whatever s
 // and c are.  NaNs are detected separately.
@@ -40,15 +41,14 @@ __device__ __forceinline__ uint32_t vbin_bits(float x, float s, float c)
 enum { M_DONE = 0, M_VH, M_VC, M_VM, M_KA, M_KH, M_KC };
 
 // Four tag bytes against the target bytes of vbx: 0x80 in each byte whose tag
-// equals its target.  Tags are < 0x80; a byte of w ^ vbx is then zero exactly
-// at a match, and for the other bytes OR-ing 0x80 keeps the per-byte
-// subtraction from borrowing across bytes.  Valid while no byte of w ^ vbx is
-// 0x80 (targets of coordinates that search nothing are 0xFF, which matches
-// only the padding tag 0x7F; callers skip such hits).
+// equals its target, 0 elsewhere.  Exact for every byte value: the sum of a
+// byte's low seven bits and 0x7F sets its top bit iff they are not all zero
+// and cannot carry into the next byte.  (Targets of coordinates that search
+// nothing are 0xFF, equal to the padding tag; callers skip such hits.)
 __device__ __forceinline__ uint32_t tag_match(uint32_t w, uint32_t vbx)
 {
-    const uint32_t t = ((w ^ vbx) | 0x80808080u) - 0x01010101u;
-    return ~t & 0x80808080u;
+    const uint32_t x = w ^ vbx;
+    return ~(((x & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | x) & 0x80808080u;
 }
 
 // Two-sum: s + e == a + b exactly (Knuth); no products, so nothing to fuse.
