@@ -84,9 +84,10 @@ typedef struct {
 } aspis_assignment;
 
 /* Outcome of detection and selection for one round; lives in device memory
- * (the caller allocates sizeof(aspis_detection) bytes).  Written by
- * aspis_detect (all but n_sel), aspis_select (n_sel) and aspis_aggregate
- * (status = ASPIS_E_EMPTY when n_sel == 0). */
+ * (the caller allocates sizeof(aspis_detection) = 36 bytes).  Written by
+ * aspis_detect (all but n_sel; n_sel and median_exact reset to 0),
+ * aspis_select (n_sel) and aspis_aggregate (status = ASPIS_E_EMPTY when
+ * n_sel == 0; median_exact added to). */
 typedef struct {
     uint32_t clique_mask;        /* the maximum clique with the smallest mask value */
     int32_t  omega;              /* size of a maximum clique */
@@ -97,6 +98,10 @@ typedef struct {
     uint32_t search_nodes;       /* Bron-Kerbosch nodes visited (diagnostic) */
     uint32_t node_budget;        /* in: node limit per search branch, 0 = default
                                     (2^20); read by aspis_detect, never written */
+    uint32_t median_exact;       /* coordinates that the lower median resolved by
+                                    its exact key-space path (a NaN, a crowded or
+                                    overflowed bin) since aspis_detect reset it;
+                                    added to by aspis_aggregate (diagnostic) */
 } aspis_detection;
 
 /* Short text for a status code. */
@@ -116,6 +121,14 @@ aspis_status aspis_assignment_to_device(aspis_assignment *a);
 
 /* Frees the host tables and the device mirror and zeroes *a. */
 void aspis_assignment_free(aspis_assignment *a);
+
+/* Bytes of device workspace the calls below need for assignment a: always 0.
+ * Every per-round intermediate is a named caller buffer (file_neq, adj, det,
+ * sel, out) and each kernel keeps its working set in shared memory, so no
+ * call takes a workspace argument.  Kept so that a caller written against a
+ * workspace-passing interface can size it (to nothing).  Host only; a NULL a
+ * also gives 0. */
+size_t aspis_workspace_bytes(const aspis_assignment *a);
 
 /* Steps 1-2: per-file agreement alpha_i and graph G (Section 4, the
  * definitions of alpha_i^{(j1,j2)} and alpha^{(j1,j2)} and the edge rule of

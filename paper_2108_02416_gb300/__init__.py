@@ -50,15 +50,16 @@ class _Assignment(ctypes.Structure):
 
 
 class Detection(ctypes.Structure):
-    """Host image of ``aspis_detection`` (32 bytes)."""
+    """Host image of ``aspis_detection`` (36 bytes)."""
     _fields_ = [("clique_mask", ctypes.c_uint32), ("omega", ctypes.c_int32),
                 ("n_max_cliques", ctypes.c_uint32), ("success", ctypes.c_int32),
                 ("n_sel", ctypes.c_int32), ("status", ctypes.c_int32),
-                ("search_nodes", ctypes.c_uint32), ("node_budget", ctypes.c_uint32)]
+                ("search_nodes", ctypes.c_uint32), ("node_budget", ctypes.c_uint32),
+                ("median_exact", ctypes.c_uint32)]
 
     @classmethod
     def from_tensor(cls, t):
-        """Read a device/host uint8[32] tensor holding an aspis_detection."""
+        """Read a device/host uint8 tensor holding an aspis_detection."""
         raw = bytes(t.detach().to("cpu").contiguous().numpy().tobytes())
         return cls.from_buffer_copy(raw)
 
@@ -115,6 +116,7 @@ def _load():
     sig = {
         "aspis_status_str": ([i32], ctypes.c_char_p),
         "aspis_abi_version": ([], i32),
+        "aspis_workspace_bytes": ([A], ctypes.c_size_t),
         "aspis_assign": ([i32, i32, A], i32),
         "aspis_assignment_to_device": ([A], i32),
         "aspis_assignment_free": ([A], None),

@@ -259,6 +259,8 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     }
     __syncthreads();
 
+    uint32_t exact_cnt = 0u;        // coordinates resolved by the exact passes (thread 0)
+
     // The previous tile ("pending"): its median bins are known, its members
     // are listed during the next sweep and ranked after it.
     bool have_p = false;
@@ -604,6 +606,11 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
 
             if (__syncthreads_or(need_general)) {
                 // ---- exact fallback passes (rare), values re-read from global memory
+                {
+                    const uint32_t md0 = tid < TC ? S(S_MODE, tid) : (uint32_t)M_DONE;
+                    const int ne = __syncthreads_count(md0 == M_VM || md0 == M_KA);
+                    if (tid == 0) exact_cnt += (uint32_t)ne;
+                }
                 auto reread = [&](int j, int k) -> uint32_t {
                     return __ldcg(reinterpret_cast<const unsigned int *>(row_ptr(lb, j)) + k);
                 };
@@ -738,6 +745,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             __syncthreads();
             rank_pending();
         }
+        if (tid == 0 && exact_cnt) atomicAdd(&det->median_exact, exact_cnt);
     }
 }
 
@@ -858,6 +866,12 @@ median_radix_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t 
         }
         if (w == 0 && live) out[col] = __uint_as_float(from_key(pre[lane]));
         __syncthreads();
+    }
+    // every coordinate of this path is resolved exactly
+    if (tid == 0) {
+        uint32_t cnt = 0u;
+        for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x) cnt += (uint32_t)min((int64_t)32, d - t * 32);
+        atomicAdd(&det->median_exact, cnt);
     }
 }
 

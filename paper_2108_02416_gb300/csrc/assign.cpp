@@ -58,7 +58,11 @@ extern "C" const char *aspis_status_str(int status)
     }
 }
 
-extern "C" int aspis_abi_version(void) { return 1; }
+extern "C" int aspis_abi_version(void) { return 2; }
+
+// No call needs device workspace: the per-round intermediates are caller
+// buffers and the kernels' working sets live in shared memory.
+extern "C" size_t aspis_workspace_bytes(const aspis_assignment *) { return 0; }
 
 extern "C" aspis_status aspis_assign(int K, int r, aspis_assignment *out)
 {

@@ -113,6 +113,7 @@ detect_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection *det)
         det->n_max_cliques = n;
         det->success = (n == 1u && !any_over) ? 1 : 0;
         det->n_sel = 0;
+        det->median_exact = 0u;
         det->status = any_over ? ASPIS_E_LIMIT : ASPIS_OK;
         det->search_nodes = total;
     }

@@ -207,6 +207,21 @@ def corrupted_mask(w: Workload, file_workers: np.ndarray) -> np.ndarray:
     return mask
 
 
+def random_graph(K: int, p: float, seed: int) -> list[int]:
+    """Neighbour masks of an Erdos-Renyi graph G(K, p): every pair (j, k)
+    is an edge with probability p, drawn from a seeded generator.  Used as a
+    clique-search input with many maximal cliques."""
+    rng = np.random.default_rng(seed)
+    coin = rng.random((K, K)) < p
+    rows = [0] * K
+    for j in range(K):
+        for k in range(j + 1, K):
+            if coin[j, k]:
+                rows[j] |= 1 << k
+                rows[k] |= 1 << j
+    return rows
+
+
 def attack_graph(w: Workload) -> list[int]:
     """Neighbour masks (bit k = worker k) of the agreement graph that the
     workload's attack leaves, for any K, without materialising the C(K,r)
@@ -314,29 +329,37 @@ def build_copies_np(w: Workload, file_workers: np.ndarray, c0: int = 0,
 
 
 def build_copies_torch(w: Workload, file_workers: np.ndarray, device, out=None,
-                       pad_value: float = 0.0):
+                       pad_value: float = 0.0, c0: int = 0, c1: int | None = None):
     """The same copies as :func:`build_copies_np`, written into a device
     tensor [f, r, ld] (allocated unless ``out`` is given).  Generation is done
-    one file at a time so the working set stays a few vectors."""
+    one file at a time so the working set stays a few vectors.  With c0/c1
+    only coordinates [c0, c1) are made (a tensor [f, r, round_up(c1 - c0,
+    ld_align)]); every value equals the one of the whole-vector build."""
     import torch
     fw = np.asarray(file_workers)
     f, r = fw.shape
-    d, ld = w.d, w.ld
+    c1 = w.d if c1 is None else c1
+    if not 0 <= c0 <= c1 <= w.d:
+        raise ValueError(f"slice [{c0}, {c1}) of d={w.d}")
+    d = c1 - c0
+    ld = w.ld if (c0, c1) == (0, w.d) else max(w.ld_align, -(-d // w.ld_align) * w.ld_align)
     if out is None:
         out = torch.empty((f, r, ld), dtype=torch.float32, device=device)
     if ld > d:
         out[:, :, d:] = pad_value
+    if d == 0:
+        return out
     mask = corrupted_mask(w, fw)
     bad = None
     if mask.any() and w.distortion in ("alie", "foe"):
-        bad = _alie_torch(w, 0, d, device)
-    b = 0.01 * normal_torch(w.seed, STREAM_B, 0, d, device)
+        bad = _alie_torch(w, c0, c1, device)
+    b = 0.01 * normal_torch(w.seed, STREAM_B, c0, c1, device)
     for i in range(f):
-        g = honest_torch(w.seed, i, 0, d, device, b)
+        g = honest_torch(w.seed, i, c0, c1, device, b)
         for s in range(r):
             if not mask[i, s]:
                 if w.copy_noise:
-                    z = normal_torch(w.seed, STREAM_COPY0 + 8 * i + s, 0, d, device)
+                    z = normal_torch(w.seed, STREAM_COPY0 + 8 * i + s, c0, c1, device)
                     out[i, s, :d].copy_((g.to(torch.float64) + w.copy_noise * z).to(torch.float32))
                 else:
                     out[i, s, :d].copy_(g)

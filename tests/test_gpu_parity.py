@@ -365,6 +365,7 @@ def _median_case(vals, r=2):
     a = ap.aspis_assign(K, r)
     buf = gpu_round(ap, torch, torch.from_numpy(host).to(DEV), d, a)
     assert_round_matches(ap, buf, want)
+    return buf
 
 
 def test_median_nan_inf_outside_sampled_rows():
@@ -484,6 +485,42 @@ def test_median_values_far_below_a_narrow_sample():
         vals[rows[:100], c] = np.float32(-9.0 - c)
         vals[rows[100:], c] = np.float32(3.0 + c)
     _median_case(vals)
+
+
+# --------------------------------- 8-bit bin counters that overflow, very large f
+
+
+@pytest.mark.parametrize("n,equal", [(455, 300), (600, 280)])
+def test_median_bin_counter_overflow(n, equal):
+    """More than 255 equal values in one bin overflow an 8-bit counter; the
+    bin search sees the coordinate's total change and the exact path decides
+    (n = 600 also takes the widened bin map of more than 512 files)."""
+    rng = np.random.default_rng(n)
+    d = 64
+    vals = rng.standard_normal((n, d)).astype(np.float32)
+    for c in range(d):
+        rows = rng.choice(np.arange(32, n), size=equal, replace=False)
+        vals[rows, c] = np.float32(0.125 + c * 1e-3)      # inside the sampled range
+    buf = _median_case(vals, r=2 if n <= 465 else 3)     # K <= 31 files
+    assert buf.detection().median_exact == d
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("layout", ["aligned", "offset1"])
+def test_round_k21_r4_near_the_file_limit(mode, layout):
+    """K=21, r=4: f = 5985 files, more than any tag layout of the median holds
+    in shared memory; the radix-select path (median) and the tag-free mean
+    take them, aligned or not."""
+    w = synth.Workload("k21r4", K=21, r=4, d=1029, q=4, attack="strong", z=1.0, seed=12)
+    buf, want, host = run_case(w, mode=mode, offset=1 if layout == "offset1" else 0)
+    if mode == 0:
+        assert_round_matches(ap, buf, want)
+        assert buf.detection().median_exact == w.d
+    else:
+        assert_round_matches(ap, buf, want, mode=1, check_out=False)
+        rows = np.array([host[i, want.sel[i], : w.d] for i in range(len(want.sel))
+                         if want.sel[i] >= 0])
+        assert_mean_close(buf.out.cpu().numpy(), want.out, np.abs(rows.astype(np.float64)).mean(0))
 
 
 # ------------------------------------------------ coordinate-split round on one GPU
