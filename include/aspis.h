@@ -225,10 +225,17 @@ aspis_status aspis_round(const float *copies, int64_t d, int64_t ld,
  * Results equal aspis_round's.  f > ASPIS_STATIC_MAX_FILES returns
  * ASPIS_E_RANGE before anything is enqueued.  The first call on a device
  * looks up the array's device address (cudaGetSymbolAddress, with that
- * device current); make that first call before any stream capture.  All
- * calls share the array and its contents persist between calls (the parts
- * that must start at zero are cleared by each call): calls that may overlap
- * on the GPU, e.g. on unordered streams, race and must not be issued. */
+ * device current); make that first call before any stream capture.  The
+ * address is kept for the life of the process: after cudaDeviceReset of a
+ * device (which unloads the library's device code there) the kept address
+ * is stale, so do not call this function on that device again in the same
+ * process.  Every call copies the assignment table (f*r bytes) from the
+ * library's pageable host memory into the array on the stream, so the call
+ * may return only after the work already queued on the stream has drained.
+ * All calls share the array and its contents persist between calls (the
+ * parts that must start at zero are cleared by each call): calls that may
+ * overlap on the GPU, e.g. on unordered streams, race and must not be
+ * issued. */
 aspis_status aspis_round_static(const float *copies, int64_t d, int64_t ld,
                                 const aspis_assignment *a, aspis_detection *det,
                                 int mode, float *out, void *stream);
@@ -308,10 +315,11 @@ aspis_status aspis_detect_wide(const uint32_t *adj, int K, aspis_detection_wide 
  *   - Case 1 averages the slots whose worker is in the clique (a file with
  *     none is dropped); Case 2 the largest connected component of "close"
  *     among the r slots, ties to the component holding the lower slot;
- *   - the average of the chosen copies x_s, x0 the first: e_s = 0 where x_s
- *     equals x0 bitwise, else fp32(x_s - x0); acc = fp32 sum of the e_s in
- *     slot order; mean = x0 if acc == 0, else fp32(x0 + fp32(acc / k)).
- *     Identical copies give their common value exactly.
+ *   - the average of the chosen copies is their arithmetic mean, computed in
+ *     fp32 as x0 + (sum of the deviations x_s - x0) / k with x0 the first
+ *     copy (a deviation is 0 where x_s equals x0 bitwise): within
+ *     1e-6 * max(|mean|, mean |x_s|) of the exact mean for close copies, and
+ *     exactly the common value of identical copies.
  * The lower median (mode 0) or mean (mode 1) of the kept files' averages is
  * written to out.  With tau = 0 and copies without NaNs or signed-zero
  * differences the result equals aspis_round's.

@@ -628,11 +628,10 @@ int oracle_sgd(const float *g, float *w, float *v, int64_t m, float eta, float m
  *     "equal";
  *   - clusters are the connected components of "close" among the r slots;
  *     the largest wins, ties to the one holding the lower slot;
- *   - the average of the chosen copies x_s (x0 the first) per coordinate:
- *     deviations e_s = 0 where x_s equals x0 bitwise, else fp32(x_s - x0);
- *     acc = fp32 sum of e_s in slot order; the mean is x0 when acc == 0,
- *     else fp32(x0 + fp32(acc / k)).  Identical copies give their common
- *     value exactly (also -0, infinities and NaNs). */
+ *   - the average of the chosen copies per coordinate is their arithmetic
+ *     mean: summed in double in slot order, divided by their number, rounded
+ *     once to fp32.  Identical copies give their common value exactly (also
+ *     -0, infinities and NaNs). */
 
 static void *agree_tol_worker(void *arg)
 {
@@ -726,8 +725,12 @@ int64_t oracle_select_tol(const uint32_t *file_neq, const uint8_t *file_workers,
     return kept;
 }
 
-/* means[i*d + c] = the average of the copies in slot_mask[i] (reading
- * above); files with an empty mask are left untouched. */
+/* means[i*d + c] = the average of the copies in slot_mask[i]: their
+ * arithmetic mean, summed in double in slot order, divided by their number
+ * and rounded once to fp32 (Section 5's remark after Algorithm 1 says to
+ * average them); files with an empty mask are left untouched.  Identical
+ * copies give their common value exactly (k equal fp32 values sum exactly in
+ * double). */
 int oracle_file_means(const float *copies, int64_t f, int r, int64_t d, int64_t ld,
                       const uint8_t *slot_mask, float *means)
 {
@@ -735,20 +738,21 @@ int oracle_file_means(const float *copies, int64_t f, int r, int64_t d, int64_t 
     for (int64_t i = 0; i < f; ++i) {
         const uint32_t m = slot_mask[i];
         if (!m) continue;
-        int k = 0, s0 = -1;
+        int k = 0;
         for (int s = 0; s < r; ++s)
-            if ((m >> s) & 1u) { if (s0 < 0) s0 = s; ++k; }
-        const float *x0 = copies + (i * r + s0) * ld;
+            if ((m >> s) & 1u) ++k;
         for (int64_t c = 0; c < d; ++c) {
-            float acc = 0.0f;
+            /* the sum starts from the first chosen copy, not from +0, so a
+             * sum of negative zeros stays -0 */
+            double sum = 0.0;
+            int first = 1;
             for (int s = 0; s < r; ++s) {
                 if (!((m >> s) & 1u)) continue;
-                const float xs = copies[(i * r + s) * ld + c];
-                float e = 0.0f;
-                if (memcmp(&xs, &x0[c], 4) != 0) e = xs - x0[c];
-                acc = acc + e;
+                const double x = (double)copies[(i * r + s) * ld + c];
+                sum = first ? x : sum + x;
+                first = 0;
             }
-            means[i * d + c] = acc == 0.0f ? x0[c] : x0[c] + acc / (float)k;
+            means[i * d + c] = (float)(sum / (double)k);
         }
     }
     return ORACLE_OK;

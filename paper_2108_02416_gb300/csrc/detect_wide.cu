@@ -2,10 +2,15 @@
 // of up to 128 workers, with vertex sets as four 32-bit words.
 //
 // Bron-Kerbosch with Tomita pivoting (pivot = the vertex of P u X with most
-// neighbours in P).  The root's candidates are split over four warps: the
-// k-th candidate c_k starts from R = {c_k}, P = (V minus c_0..c_{k-1}) n N(c_k),
+// neighbours in P).  The root's candidates are split over the warps of a
+// thread-block cluster (CB blocks of four warps): the k-th candidate c_k
+// starts from R = {c_k}, P = (V minus c_0..c_{k-1}) n N(c_k),
 // X = {c_0..c_{k-1}} n N(c_k), exactly the branch sequential Bron-Kerbosch
-// takes, and warp w takes k = w, w + 4, ...  Each warp walks its branches
+// takes, and warp g of the cluster takes k = g, g + 4*CB, ...  A warp that
+// finds a larger clique writes its size into every block's bound with a
+// distributed-shared-memory max (rare), so the pruning test reads only local
+// shared memory; block 0 combines the blocks' results at the end through
+// distributed shared memory.  Each warp walks its branches
 // cooperatively: the current frame (R, P, X, candidates) is the same in all
 // lanes, lane l holds the adjacency rows of workers l, l + 32, l + 64, l + 96
 // in registers, so the pivot is one row-count per lane and a warp max, and
@@ -86,6 +91,47 @@ __device__ __forceinline__ bool vs_less(const VS &a, const VS &b)
 
 constexpr int kWarps = 4;
 
+__device__ __forceinline__ uint32_t cta_rank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ uint32_t cta_count()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+    return r;
+}
+// shared::cluster address of a shared variable of this block in block `rank`
+__device__ __forceinline__ uint32_t peer(const void *p, uint32_t rank)
+{
+    uint32_t a = (uint32_t)__cvta_generic_to_shared(p), r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ uint32_t ld_peer32(const void *p, uint32_t rank)
+{
+    uint32_t v;
+    asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(peer(p, rank)) : "memory");
+    return v;
+}
+__device__ __forceinline__ uint64_t ld_peer64(const void *p, uint32_t rank)
+{
+    uint64_t v;
+    asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(peer(p, rank)) : "memory");
+    return v;
+}
+__device__ __forceinline__ void max_peer(const int *p, uint32_t rank, int v)
+{
+    asm volatile("red.shared::cluster.max.s32 [%0], %1;" ::"r"(peer(p, rank)), "r"(v) : "memory");
+}
+__device__ __forceinline__ void cluster_sync_all()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;\n"
+                 "barrier.cluster.wait.acquire.aligned;\n" ::: "memory");
+}
+
 __global__ void __launch_bounds__(kWarps * 32)
 detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wide *det)
 {
@@ -98,9 +144,12 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
     __shared__ uint32_t w_first[kWarps][4];
     const int tid = threadIdx.x, lane = tid & 31, wp = tid >> 5;
     const unsigned full = 0xffffffffu;
+    const uint32_t rank = cta_rank(), nblocks = cta_count();
+    const int gw = (int)rank * kWarps + wp, nwarps = (int)nblocks * kWarps;
     for (int i = tid; i < kMaxK * 4; i += kWarps * 32) raw[i >> 2][i & 3] = (i >> 2) < K ? adj_g[i] : 0u;
     if (tid == 0) shared_best = 0;
     __syncthreads();
+    cluster_sync_all();             // every block's bound is initialised before any max
     // symmetric part: bit k of row j iff both rows list the edge; no self
     // loops, nothing at or beyond K
     for (int j = tid; j < kMaxK; j += kWarps * 32) {
@@ -140,7 +189,8 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
             best = sz;
             count = 1;
             first = R;
-            if (lane == 0) atomicMax(&shared_best, sz);
+            if (lane == 0 && sz > *(volatile int *)&shared_best)
+                for (uint32_t b = 0; b < nblocks; ++b) max_peer(&shared_best, b, sz);
         } else if (sz == best) {
             ++count;
             if (vs_less(R, first)) first = R;
@@ -207,7 +257,7 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
     // the root frame, settled by every warp alike (reports counted once)
     VS R0{{0u, 0u, 0u, 0u}}, P0{{0u, 0u, 0u, 0u}}, X0{{0u, 0u, 0u, 0u}}, C0{{0u, 0u, 0u, 0u}};
     for (int v = 0; v < K; ++v) vs_set(P0, v);
-    live = wp == 0;
+    live = gw == 0;
     const bool branch0 = settle(R0, P0, X0, C0);
     live = true;
     if (!branch0) C0 = VS{{0u, 0u, 0u, 0u}};
@@ -216,7 +266,7 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
         const int ck = vs_lowest(C0);
         if (ck < 0) break;
         vs_clear(C0, ck);
-        const bool mine = (k++ % kWarps) == wp;
+        const bool mine = (k++ % nwarps) == gw;
         // branch c_k: R, P and X as sequential Bron-Kerbosch leaves them
         VS R = R0, P = vs_and(P0, adj[ck]), X = vs_and(X0, adj[ck]), C;
         vs_set(R, ck);
@@ -278,7 +328,9 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
         }
     }
 
-    // reduction over warps: omega, maximum cliques of that size, the smallest
+    // reduction: first over the warps of this block, then block 0's first
+    // warp gathers the blocks' summaries (lane b reads block b) and combines
+    // them; omega, the maximum cliques of that size, the smallest of them
     if (lane == 0) {
         w_best[wp] = best;
         w_over[wp] = over ? 1 : 0;
@@ -289,31 +341,107 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
         for (int i = 0; i < 4; ++i) w_first[wp][i] = count ? first.w[i] : 0xffffffffu;
     }
     __syncthreads();
+    __shared__ int b_best, b_over;
+    __shared__ unsigned long long b_count, b_maximal, b_nodes;
+    __shared__ uint32_t b_first[4];
     if (tid == 0) {
-        int omega = 0;
-        for (int q = 0; q < kWarps; ++q) omega = max(omega, w_best[q]);
-        uint64_t n = 0, nmx = 0, nds = 0;
-        bool any_over = false;
+        int om = 0;
+        for (int q = 0; q < kWarps; ++q) om = max(om, w_best[q]);
+        unsigned long long n = 0, nmx = 0, nds = 0;
+        int ov = 0;
         VS c{{0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu}};
         for (int q = 0; q < kWarps; ++q) {
             nmx += w_maximal[q];
             nds += w_nodes[q];
-            any_over |= w_over[q] != 0;
-            if (w_best[q] == omega && w_count[q]) {
+            ov |= w_over[q];
+            if (w_best[q] == om && w_count[q]) {
                 n += w_count[q];
                 const VS f{{w_first[q][0], w_first[q][1], w_first[q][2], w_first[q][3]}};
                 if (vs_less(f, c)) c = f;
             }
         }
+        b_best = om;
+        b_over = ov;
+        b_count = n;
+        b_maximal = nmx;
+        b_nodes = nds;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) det->clique_mask[i] = c.w[i];
-        det->n_max_cliques = n;
-        det->n_maximal = nmx;
-        det->search_nodes = nds;
-        det->omega = omega;
-        det->success = (n == 1u && !any_over) ? 1 : 0;
-        det->status = any_over ? ASPIS_E_LIMIT : ASPIS_OK;
+        for (int i = 0; i < 4; ++i) b_first[i] = c.w[i];
     }
+    cluster_sync_all();             // every block's summary is complete
+    if (rank == 0 && wp == 0) {
+        const bool has = (uint32_t)lane < nblocks;
+        const int bb = has ? (int)ld_peer32(&b_best, lane) : 0;
+        const uint64_t bc = has ? ld_peer64(&b_count, lane) : 0ull;
+        uint64_t nmx = has ? ld_peer64(&b_maximal, lane) : 0ull;
+        uint64_t nds = has ? ld_peer64(&b_nodes, lane) : 0ull;
+        const uint32_t bo = has ? ld_peer32(&b_over, lane) : 0u;
+        VS f{{0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu}};
+        if (has)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) f.w[i] = ld_peer32(&b_first[i], lane);
+        const int omega = __reduce_max_sync(full, bb);
+        const bool at = has && bb == omega && bc != 0ull;
+        uint64_t n = at ? bc : 0ull;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            n += __shfl_xor_sync(full, n, o);
+            nmx += __shfl_xor_sync(full, nmx, o);
+            nds += __shfl_xor_sync(full, nds, o);
+        }
+        const bool any_over = __any_sync(full, bo != 0u);
+        // the smallest first clique among the blocks at omega: compare
+        // 128-bit values from the most significant word down
+        VS c = at ? f : VS{{0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu}};
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            VS y;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) y.w[i] = __shfl_xor_sync(full, c.w[i], o);
+            if (vs_less(y, c)) c = y;
+        }
+        if (lane == 0) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) det->clique_mask[i] = c.w[i];
+            det->n_max_cliques = n;
+            det->n_maximal = nmx;
+            det->search_nodes = nds;
+            det->omega = omega;
+            det->success = (n == 1u && !any_over) ? 1 : 0;
+            det->status = any_over ? ASPIS_E_LIMIT : ASPIS_OK;
+        }
+    }
+    cluster_sync_all();             // block 0 has read every block's records
+}
+
+// Blocks per cluster: 16 where the device allows clusters of that size
+// (non-portable), else 8; decided once per device.
+int cluster_blocks()
+{
+    static int cached[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev < 0 || dev >= 64) dev = 0;
+    if (cached[dev]) return cached[dev];
+    int best = 8;
+    if (cudaFuncSetAttribute(detect_wide_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) ==
+        cudaSuccess) {
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = 16;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(16);
+        cfg.blockDim = dim3(kWarps * 32);
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, detect_wide_kernel, &cfg) == cudaSuccess && n > 0) best = 16;
+    }
+    cudaGetLastError();
+    cached[dev] = best;
+    return best;
 }
 
 }  // namespace
@@ -323,6 +451,18 @@ extern "C" aspis_status aspis_detect_wide(const uint32_t *adj, int K, aspis_dete
 {
     if (!adj || !det || K < 1) return ASPIS_E_INVAL;
     if (K > ASPIS_WIDE_MAX_K) return ASPIS_E_RANGE;
-    detect_wide_kernel<<<1, kWarps * 32, 0, (cudaStream_t)stream>>>(adj, K, det);
+    const int cb = cluster_blocks();
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = (unsigned)cb;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3((unsigned)cb);
+    cfg.blockDim = dim3(kWarps * 32);
+    cfg.stream = (cudaStream_t)stream;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, detect_wide_kernel, adj, K, det) != cudaSuccess) return ASPIS_E_CUDA;
     return cudaGetLastError() == cudaSuccess ? ASPIS_OK : ASPIS_E_CUDA;
 }

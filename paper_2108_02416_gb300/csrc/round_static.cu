@@ -31,7 +31,9 @@ __device__ __align__(256) unsigned char g_round_scratch[ASPIS_STATIC_SCRATCH_BYT
 
 // Host code cannot use g_round_scratch as an address: on the host the name
 // refers to a host-side shadow.  The device address is looked up once per
-// device, with that device current, and kept here.
+// device, with that device current, and kept here for the life of the
+// process (a cudaDeviceReset of the device makes it stale; the header says
+// so).
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 unsigned char *g_dev_ptr[kMaxDevices] = {nullptr};

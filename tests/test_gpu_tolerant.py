@@ -1,6 +1,8 @@
 """The round for copies that are not bit-identical (aspis_round_tolerant)
-against the oracle: mismatch words, graph, clique, slot masks, the kept
-files' averages and the median, bit for bit; the mean within its tolerance.
+against the oracle: mismatch words, graph, clique and slot masks bit for bit;
+the kept files' averages, and the median and mean over them, within
+1e-6 * max(|oracle|, mean |copy|) + 1e-30 of the oracle's arithmetic means
+(the kernel averages in fp32).
 Cases: tau = 0 on bit-identical copies (equal to the exact round), honest
 copies with per-copy noise below tau under the weak, optimal and
 all-adversary attacks (Case 1 averages, Case 2 clusters, r = 2 to 6), the
@@ -38,7 +40,7 @@ def run(host, w, tau, mode=0, offset=0, ldm_pad=0):
     return buf
 
 
-def check(buf, want, mode=0, kept_scale=None):
+def check(buf, want, host, mode=0, exact_means=False):
     det = buf.detection()
     assert det.status == ap.OK, ap.status_str(det.status)
     assert np.array_equal(as_u32(buf.file_neq), want.file_neq), "file_neq"
@@ -52,11 +54,36 @@ def check(buf, want, mode=0, kept_scale=None):
     d = want.means.shape[1]
     kept = mask != 0
     means = buf.means[:, :d].cpu().numpy()
-    assert np.array_equal(means[kept].view(np.uint32), want.means[kept].view(np.uint32)), "averages"
+    # per kept file and coordinate: max(|average|, mean |chosen copy|)
+    scale = np.fmax(np.abs(want.means[kept].astype(np.float64)), chosen_abs_mean(host, want)[kept])
+    scale = np.where(np.isnan(scale), 0.0, scale)       # NaN copies: compared as NaN below
+    err = np.abs(means[kept].astype(np.float64) - want.means[kept].astype(np.float64))
+    bad = ~(err <= 1e-6 * scale + 1e-30) & ~(np.isnan(means[kept]) & np.isnan(want.means[kept]))
+    assert not bad.any(), f"averages differ at {np.argwhere(bad)[:5]}"
+    # an order statistic moves by at most the largest change of its inputs
+    col_scale = scale.max(axis=0) if scale.size else np.zeros(d)
+    got = buf.out.cpu().numpy().astype(np.float64)
+    ref = want.out.astype(np.float64)
     if mode == 0:
-        assert np.array_equal(as_u32(buf.out), want.out.view(np.uint32)), "lower median"
+        err = np.abs(got - ref)
+        bad = ~(err <= 1e-6 * col_scale + 1e-30) & ~(np.isnan(got) & np.isnan(ref))
+        assert not bad.any(), f"lower median differs at {np.nonzero(bad)[0][:5]}"
+        if exact_means:
+            assert np.array_equal(as_u32(buf.out), want.out.view(np.uint32)), "lower median bits"
     else:
-        assert_mean_close(buf.out.cpu().numpy(), want.out, np.abs(want.means[kept]).mean(axis=0))
+        assert_mean_close(buf.out.cpu().numpy(), want.out, col_scale)
+
+
+def chosen_abs_mean(host, want):
+    """[f, d] mean |x| over the chosen copies of each file (0 where dropped)."""
+    f, r, _ = host.shape
+    d = want.means.shape[1]
+    out = np.zeros((f, d))
+    for i in range(f):
+        slots = [s for s in range(r) if (int(want.slot_mask[i]) >> s) & 1]
+        if slots:
+            out[i] = np.abs(host[i, slots, :d].astype(np.float64)).mean(axis=0)
+    return out
 
 
 CASES = [
@@ -80,7 +107,8 @@ def test_tolerant_round(name, d, noise, tau, mode):
     oa = oracle.assign(w.K, w.r)
     host = synth.build_copies_np(w, oa.file_workers)
     want = oracle.run_round_tolerant(host, oa, tau, w.d, mode)
-    check(run(host, w, tau, mode), want, mode)
+    # identical copies average to themselves on both sides: the median is exact
+    check(run(host, w, tau, mode), want, host, mode, exact_means=noise == 0.0)
     if noise == 0.0 and tau == 0.0 and mode == 0:
         exact = oracle.run_round(host, oa, w.d, 0)
         assert np.array_equal(want.out.view(np.uint32), exact.out.view(np.uint32))
@@ -93,7 +121,7 @@ def test_tolerant_unaligned_paths(offset, ldm_pad):
     oa = oracle.assign(w.K, w.r)
     host = synth.build_copies_np(w, oa.file_workers)
     want = oracle.run_round_tolerant(host, oa, 1e-4, w.d, 0)
-    check(run(host, w, 1e-4, 0, offset, ldm_pad), want, 0)
+    check(run(host, w, 1e-4, 0, offset, ldm_pad), want, host, 0)
 
 
 @pytest.mark.parametrize("K,r,q,attack", [(6, 2, 2, "weak"), (8, 2, 3, "strong"), (8, 4, 3, "strong"),
@@ -104,7 +132,7 @@ def test_tolerant_other_r(K, r, q, attack):
     oa = oracle.assign(w.K, w.r)
     host = synth.build_copies_np(w, oa.file_workers)
     want = oracle.run_round_tolerant(host, oa, 1e-4, w.d, 0)
-    check(run(host, w, 1e-4), want)
+    check(run(host, w, 1e-4), want, host)
 
 
 def test_tolerant_foe_and_nans():
@@ -113,11 +141,11 @@ def test_tolerant_foe_and_nans():
     oa = oracle.assign(w.K, w.r)
     host = synth.build_copies_np(w, oa.file_workers)
     want = oracle.run_round_tolerant(host, oa, 1e-4, w.d, 0)
-    check(run(host, w, 1e-4), want)
+    check(run(host, w, 1e-4), want, host)
     host[3, 1, 5] = np.nan                     # one copy is no longer close to anything
     host[10, :, 7] = np.nan                    # identical NaNs are not close either
     want = oracle.run_round_tolerant(host, oa, 1e-4, w.d, 0)
-    check(run(host, w, 1e-4), want)
+    check(run(host, w, 1e-4), want, host)
 
 
 def test_tolerant_rejects_bad_tau():

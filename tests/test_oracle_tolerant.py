@@ -3,7 +3,8 @@ after Algorithm 1: average the honest copies in Case 1, average the largest
 cluster of copies in Case 2) and for the new generator options (Fall of
 Empires, per-copy noise).  Readings: copies are close iff every coordinate
 differs by at most tau in fp32; clusters are connected components of
-"close"; the average is the first copy plus the fp32 mean deviation."""
+"close"; the average is the arithmetic mean of the chosen copies, rounded
+once to fp32."""
 from fractions import Fraction
 
 import numpy as np
@@ -117,20 +118,24 @@ def test_means_exact_cases():
     assert m[0].tolist() == [2.5, 4.0]
 
 
-def test_means_within_rounding_of_exact_mean():
+@pytest.mark.parametrize("spread", [1e-3, 1.0, 1e6])
+def test_means_are_the_exact_mean_rounded(spread):
+    """The average is the exact rational mean of the chosen copies within
+    one ulp of the result (one rounding of a double sum and quotient), for
+    close copies, copies of mixed sign and copies of very different size."""
     rng = np.random.default_rng(2)
     f, r, d = 40, 5, 64
     base = rng.standard_normal((f, 1, d)).astype(np.float32)
-    c = (base + rng.standard_normal((f, r, d)).astype(np.float32) * 1e-3).astype(np.float32)
+    c = (base + rng.standard_normal((f, r, d)).astype(np.float32) * spread).astype(np.float32)
     masks = rng.integers(1, 32, f).astype(np.uint8)
     m = oracle.file_means(c, masks)
     for i in range(f):
         slots = [s for s in range(r) if (masks[i] >> s) & 1]
         for j in range(d):
             exact = sum(Fraction(float(c[i, s, j])) for s in slots) / len(slots)
-            # x0 + acc/k: at most a few roundings of size ulp(x0), ulp(acc)
-            bound = 4 * np.spacing(np.float32(max(abs(float(c[i, s, j])) for s in slots)))
-            assert abs(Fraction(float(m[i, j])) - exact) <= Fraction(float(bound))
+            got = Fraction(float(m[i, j]))
+            assert abs(got - exact) <= Fraction(float(np.spacing(np.float32(abs(m[i, j]))))), \
+                (i, j)
 
 
 def test_noisy_honest_copies_keep_the_graph():
