@@ -56,9 +56,11 @@ constexpr int kListWords = 4096;          // member lists: 32, 64 or 128 per coo
 
 // per-coordinate state, arrays of TC words
 enum { S_MIN, S_MAX, S_NAN, S_LCNT, S_MODE, S_BIN, S_REM, S_CNT, S_LO, S_HI, S_PCNT, S_PREM,
-       kStateWords };
+       S_FILT, kStateWords };
 // S_PCNT / S_PREM: count and rank of the listed bin of the pending tile
-// (S_PCNT = 0: nothing to rank for that coordinate)
+// (S_PCNT = 0: nothing to rank for that coordinate).  S_FILT: the exact
+// passes of this coordinate search inside its value bin, whose members are
+// the values whose tag byte is the bin (only they are re-read).
 
 template <int V> struct Vec;
 template <> struct Vec<4> { using T = uint4; };
@@ -103,15 +105,16 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
 
-// ascending bitonic sorting network over 16 registers
-__device__ __forceinline__ void sort16(uint32_t (&y)[16])
+// ascending bitonic sorting network over N registers (N a power of two)
+template <int N>
+__device__ __forceinline__ void sort_net(uint32_t (&y)[N])
 {
 #pragma unroll
-    for (int k = 2; k <= 16; k <<= 1)
+    for (int k = 2; k <= N; k <<= 1)
 #pragma unroll
         for (int j = k >> 1; j > 0; j >>= 1)
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
+            for (int i = 0; i < N; ++i) {
                 const int l = i ^ j;
                 if (l > i) {
                     const uint32_t a = y[i], b = y[l];
@@ -120,6 +123,22 @@ __device__ __forceinline__ void sort16(uint32_t (&y)[16])
                     y[l] = up ? max(a, b) : min(a, b);
                 }
             }
+}
+
+// the 32 values of a warp (one per lane) sorted ascending across the lanes
+// (bitonic: lane i meets lane i ^ j; the lower lane of an ascending block
+// keeps the minimum)
+__device__ __forceinline__ uint32_t warp_sort32(uint32_t x, int lane)
+{
+#pragma unroll
+    for (int k = 2; k <= 32; k <<= 1)
+#pragma unroll
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            const uint32_t y = __shfl_xor_sync(0xffffffffu, x, j);
+            const bool up = (lane & k) == 0, lower = (lane & j) == 0;
+            x = lower == up ? min(x, y) : max(x, y);
+        }
+    return x;
 }
 
 // flag |= 1 if any of a, b, c, e is NaN (one compare per pair)
@@ -192,6 +211,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     uint32_t *st = reinterpret_cast<uint32_t *>(smem + L.state);      // [kStateWords][TC]
     uint16_t *rows = reinterpret_cast<uint16_t *>(smem + L.rows);
     __shared__ int warp_tot[kWarps];
+    __shared__ int long_lists;          // some listed bin of the pending tile holds more than 8
 
     const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
     const unsigned full = 0xffffffffu;
@@ -227,6 +247,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     const int64_t ntiles = (d + TC - 1) / TC;
     const uint64_t ldb = (uint64_t)ld * 4u;                          // row pitch in bytes
 
+    if (tid == 0) long_lists = 0;
     for (int i = tid; i < TC; i += kThreads) {
         S(S_MIN, i) = 0xffffffffu;
         S(S_MAX, i) = 0u;
@@ -299,38 +320,47 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
         cp_async_commit();
     };
 
-    // Rank the pending tile's listed bins.  Lists of at most 16 keys (the
+    // Rank the pending tile's listed bins.  Lists of at most 8 keys (the
     // common case): one thread per coordinate sorts them in registers.
-    // Longer lists: kThreads/TC threads per coordinate, each counting, for its
-    // candidates, the listed keys below and at them.
+    // Longer lists: one warp per coordinate, a warp-wide sort for up to 32
+    // keys, else every lane counting, for its candidates, the listed keys
+    // below and at them.
     auto rank_pending = [&]() {
         for (int c = tid; c < TC; c += kThreads) {
             const uint32_t cnt = S(S_PCNT, c);
-            if (cnt == 0u || cnt > 16u) continue;
+            if (cnt == 0u || cnt > 8u) continue;
             const uint32_t rk = S(S_PREM, c);
-            uint32_t y[16];
+            uint32_t y[8];
 #pragma unroll
-            for (int e = 0; e < 16; ++e) y[e] = (uint32_t)e < cnt ? to_key(list[e * TC + c]) : 0xffffffffu;
-            sort16(y);
+            for (int e = 0; e < 8; ++e) y[e] = (uint32_t)e < cnt ? to_key(list[e * TC + c]) : 0xffffffffu;
+            sort_net<8>(y);
             uint32_t res = y[0];
 #pragma unroll
-            for (int e = 1; e < 16; ++e) res = (uint32_t)e == rk ? y[e] : res;
+            for (int e = 1; e < 8; ++e) res = (uint32_t)e == rk ? y[e] : res;
             out[c0_p + c] = __uint_as_float(from_key(res));
         }
-        constexpr int P = kThreads / TC;
-        const int c = tid % TC, e0 = tid / TC;
-        const uint32_t cnt = e0 < P ? S(S_PCNT, c) : 0u;
-        if (cnt <= 16u) return;
-        const uint32_t rk = S(S_PREM, c);
-        for (uint32_t e = (uint32_t)e0; e < cnt; e += P) {
-            const uint32_t x = to_key(list[e * TC + c]);
-            uint32_t lt = 0u, le = 0u;
-            for (uint32_t t2 = 0; t2 < cnt; ++t2) {
-                const uint32_t y = to_key(list[t2 * TC + c]);
-                lt += y < x;
-                le += y <= x;
+        if (!long_lists) return;
+        for (int c = w; c < TC; c += kWarps) {
+            const uint32_t cnt = S(S_PCNT, c);               // the same in every lane
+            if (cnt <= 8u) continue;
+            const uint32_t rk = S(S_PREM, c);
+            if (cnt <= 32u) {
+                const uint32_t x = warp_sort32((uint32_t)lane < cnt ? to_key(list[lane * TC + c])
+                                                                     : 0xffffffffu, lane);
+                const uint32_t res = __shfl_sync(full, x, (int)rk);
+                if (lane == 0) out[c0_p + c] = __uint_as_float(from_key(res));
+                continue;
             }
-            if (lt <= rk && rk < le) out[c0_p + c] = __uint_as_float(from_key(x));
+            for (uint32_t e = (uint32_t)lane; e < cnt; e += 32u) {
+                const uint32_t x = to_key(list[e * TC + c]);
+                uint32_t lt = 0u, le = 0u;
+                for (uint32_t t2 = 0; t2 < cnt; ++t2) {
+                    const uint32_t y = to_key(list[t2 * TC + c]);
+                    lt += y < x;
+                    le += y <= x;
+                }
+                if (lt <= rk && rk < le) out[c0_p + c] = __uint_as_float(from_key(x));
+            }
         }
     };
 
@@ -511,6 +541,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 }
             }
             __syncthreads();                                        // (R)
+            if (tid == 0) long_lists = 0;          // read by every thread before (R)
             for (int c = tid; c < TC; c += kThreads) S(S_LCNT, c) = 0u;
 
             // ---- B1: per-warp partial sums over bins [kBPW*w, kBPW*w + kBPW);
@@ -559,11 +590,18 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     int bin = min(owner * kBPW + kBPW, kVB) - 1;
                     uint32_t cnt = 0u;
                     bool f2 = false;
-                    for (int b = owner * kBPW; b < min(owner * kBPW + kBPW, kVB); ++b) {
-                        const uint32_t cb = (h[b * 32] >> shf) & msk;
+                    uint32_t cbs[kBPW];                        // the owner's bins, loaded at once
+#pragma unroll
+                    for (int i = 0; i < kBPW; ++i) {
+                        const int b = owner * kBPW + i;
+                        cbs[i] = b < kVB ? (h[b * 32] >> shf) & msk : 0u;
+                    }
+#pragma unroll
+                    for (int i = 0; i < kBPW; ++i) {
+                        const uint32_t cb = cbs[i];
                         const bool hit = !f2 && rem < cb;
                         if (hit) {
-                            bin = b;
+                            bin = owner * kBPW + i;
                             cnt = cb;
                         }
                         if (!f2 && !hit) rem -= cb;
@@ -580,6 +618,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     pc = vcm ? cnt : 0u;
                 }
                 S(S_PCNT, c) = pc;
+                if (pc > 8u) long_lists = 1;
             }
             __syncthreads();                                        // (E)
             for (int i = tid * 4; i < HW; i += kThreads * 4)
@@ -608,6 +647,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 // ---- exact fallback passes (rare), values re-read from global memory
                 {
                     const uint32_t md0 = tid < TC ? S(S_MODE, tid) : (uint32_t)M_DONE;
+                    if (tid < TC) S(S_FILT, tid) = 0u;
                     const int ne = __syncthreads_count(md0 == M_VM || md0 == M_KA);
                     if (tid == 0) exact_cnt += (uint32_t)ne;
                 }
@@ -627,31 +667,70 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                             const int sh = bits > kLogNB ? bits - kLogNB : 0;
                             const uint32_t vb = S(S_BIN, c);
                             const uint8_t *tb = reinterpret_cast<const uint8_t *>(tags);
+                            // inside a value bin only its members (tag == bin) are read
+                            const bool filt = md == M_VM || S(S_FILT, c) != 0u;
                             uint32_t a = 0xffffffffu, bmax = 0u;
-                            for (int j0 = 0; j0 < nmine; j0 += 8) {
-                                uint32_t vals[8];
-#pragma unroll
-                                for (int u = 0; u < 8; ++u)        // eight loads in flight
-                                    if (j0 + u < nmine) vals[u] = reread(j0 + u, k);
-#pragma unroll
-                                for (int u = 0; u < 8; ++u) {
-                                    const int j = j0 + u;
-                                    if (j >= nmine) break;
-                                    if (md == M_VM) {
-                                        const int q = j / RPW, p = (j % RPW) * V + k;
-                                        if (tb[((q * kWarps + w) * 32 + lane) * 4 + p] != vb) continue;
+                            if (filt) {
+                                // the members' rows from the tag bytes first, then
+                                // their loads, four at a time
+                                for (int j0 = 0; j0 < nmine; j0 += 32) {
+                                    uint32_t m = 0u;
+                                    for (int u = 0; u < 32 && j0 + u < nmine; ++u) {
+                                        const int j = j0 + u, q = j / RPW, p = (j % RPW) * V + k;
+                                        if (tb[((q * kWarps + w) * 32 + lane) * 4 + p] == vb) m |= 1u << u;
                                     }
-                                    const uint32_t key = to_key(vals[u]);
-                                    if (md == M_VM || md == M_KA) {
-                                        a = min(a, key);
-                                        bmax = max(bmax, key);
-                                    } else if (key - lo <= W) {
-                                        if (md == M_KH) {
-                                            atomicAdd(hist + (((key - lo) >> sh) * NP + k / 2) * 32 + lane,
-                                                      (k & 1) ? 0x10000u : 1u);
-                                        } else {
-                                            const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
-                                            if (at < (uint32_t)CAP) list[at * TC + c] = key;
+                                    while (m) {
+                                        uint32_t vals[4], ok = 0u;
+#pragma unroll
+                                        for (int u = 0; u < 4; ++u) {
+                                            vals[u] = 0u;
+                                            if (m) {
+                                                vals[u] = reread(j0 + __ffs(m) - 1, k);
+                                                m &= m - 1u;
+                                                ok |= 1u << u;
+                                            }
+                                        }
+#pragma unroll
+                                        for (int u = 0; u < 4; ++u) {
+                                            if (!((ok >> u) & 1u)) continue;
+                                            const uint32_t key = to_key(vals[u]);
+                                            if (md == M_VM) {
+                                                a = min(a, key);
+                                                bmax = max(bmax, key);
+                                            } else if (key - lo <= W) {
+                                                if (md == M_KH) {
+                                                    atomicAdd(hist + (((key - lo) >> sh) * NP + k / 2) * 32 + lane,
+                                                              (k & 1) ? 0x10000u : 1u);
+                                                } else {
+                                                    const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
+                                                    if (at < (uint32_t)CAP) list[at * TC + c] = key;
+                                                }
+                                            }
+                                        }
+                                    }
+                                }
+                            } else {
+                                for (int j0 = 0; j0 < nmine; j0 += 8) {
+                                    uint32_t vals[8];
+#pragma unroll
+                                    for (int u = 0; u < 8; ++u)    // eight loads in flight
+                                        if (j0 + u < nmine) vals[u] = reread(j0 + u, k);
+#pragma unroll
+                                    for (int u = 0; u < 8; ++u) {
+                                        const int j = j0 + u;
+                                        if (j >= nmine) break;
+                                        const uint32_t key = to_key(vals[u]);
+                                        if (md == M_KA) {
+                                            a = min(a, key);
+                                            bmax = max(bmax, key);
+                                        } else if (key - lo <= W) {
+                                            if (md == M_KH) {
+                                                atomicAdd(hist + (((key - lo) >> sh) * NP + k / 2) * 32 + lane,
+                                                          (k & 1) ? 0x10000u : 1u);
+                                            } else {
+                                                const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
+                                                if (at < (uint32_t)CAP) list[at * TC + c] = key;
+                                            }
                                         }
                                     }
                                 }
@@ -676,6 +755,8 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                             if (md == M_KA) {
                                 rk = krank;
                                 cnt = (uint32_t)n;
+                            } else {
+                                S(S_FILT, c) = 1u;             // [lo, hi] lies inside the value bin
                             }
                             nm = lo == hi ? M_DONE : (cnt <= (uint32_t)CAP ? M_KC : M_KH);
                         } else if (md == M_KH) {
