@@ -340,7 +340,7 @@ aspis_status aspis_round_tolerant(const float *copies, int64_t d, int64_t ld,
 
 /* The model update that follows the aggregation (Section 2, Eq. 1, with
  * the aggregate of Algorithm 1 in place of the batch gradient), with the
- * heavy-ball momentum of the experiments (Appendix B: momentum 0.9).  For
+ * heavy-ball momentum of the experiments (Appendix A.3: momentum 0.9).  For
  * every coordinate c < d:
  *     mu != 0:  v[c] <- RN(mu * v[c] + g[c]);  w[c] <- RN(w[c] - eta * v[c])
  *     mu == 0:  w[c] <- RN(w[c] - eta * g[c])   (Eq. 1; v is not touched)

@@ -23,7 +23,7 @@
  *   oracle_lower_median        coordinate-wise median of the chosen gradients (Algorithm 1, Case 2)
  *   oracle_mean                average of the chosen gradients (Algorithm 1, Case 1)
  *   oracle_sgd                 the model update with the aggregate (Section 2, Eq. 1;
- *                              Algorithm 1), with heavy-ball momentum (Appendix B)
+ *                              Algorithm 1), with heavy-ball momentum (Appendix A.3)
  *   oracle_file_agreement_tol, oracle_select_tol, oracle_file_means
  *                              the variant for copies that are not bit-identical
  *                              (Section 5, after Algorithm 1: average the honest
@@ -595,7 +595,7 @@ int oracle_mean(const float *vals, int64_t n, int64_t m, float *out)
 /* One model update with the aggregated gradient g, over m coordinates.
  * Eq. 1 (Section 2) moves w against the batch gradient with step eta; the
  * PS of Algorithm 1 uses the aggregate of the chosen copies in its place.
- * The experiments add momentum 0.9 (Appendix B), read as heavy-ball
+ * The experiments add momentum 0.9 (Appendix A.3), read as heavy-ball
  * momentum:
  *     v[c] <- mu * v[c] + g[c]        then        w[c] <- w[c] - eta * v[c],
  * each the exact real value rounded once to fp32 (C99 fmaf is exactly

@@ -1,7 +1,7 @@
 // aspis_sgd: the model update that follows the aggregation.  Eq. 1
 // (Section 2) moves the parameters against the batch gradient with step
 // eta_t; the PS of Algorithm 1 uses the aggregate of the chosen copies in its
-// place, and the experiments add momentum 0.9 (Appendix B), read as
+// place, and the experiments add momentum 0.9 (Appendix A.3), read as
 // heavy-ball momentum without dampening:
 //     v <- mu * v + g,    w <- w - eta * v,
 // each result the exact value rounded once to fp32 (one fused multiply-add).
