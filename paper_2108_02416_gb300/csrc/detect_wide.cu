@@ -2,25 +2,30 @@
 // of up to 128 workers, with vertex sets as four 32-bit words.
 //
 // Bron-Kerbosch with Tomita pivoting (pivot = the vertex of P u X with most
-// neighbours in P).  The root's candidates are split over the warps of a
-// thread-block cluster (CB blocks of four warps): the k-th candidate c_k
-// starts from R = {c_k}, P = (V minus c_0..c_{k-1}) n N(c_k),
+// neighbours in P), spread over the warps of a thread-block cluster (CB
+// blocks of four warps) in two levels.  Level 1: the k-th candidate c_k of
+// the root starts from R = {c_k}, P = (V minus c_0..c_{k-1}) n N(c_k),
 // X = {c_0..c_{k-1}} n N(c_k), exactly the branch sequential Bron-Kerbosch
-// takes, and warp g of the cluster takes k = g, g + 4*CB, ...  A warp that
-// finds a larger clique writes its size into every block's bound with a
-// distributed-shared-memory max (rare), so the pruning test reads only local
-// shared memory; block 0 combines the blocks' results at the end through
-// distributed shared memory.  Each warp walks its branches
-// cooperatively: the current frame (R, P, X, candidates) is the same in all
-// lanes, lane l holds the adjacency rows of workers l, l + 32, l + 64, l + 96
-// in registers, so the pivot is one row-count per lane and a warp max, and
-// parent frames wait on a stack in shared memory (at most K deep: every push
-// adds one worker to R).  Workers of P adjacent to all the rest of P are in
-// every maximal clique of their branch and move to R without branching, so
-// the long chains of nearly complete agreement graphs take one step.  Detection mode prunes a child whose |R| + |P|
-// cannot reach the largest clique any warp has found; enumeration mode
-// (ASPIS_WIDE_ALL_MAXIMAL) prunes nothing and counts every maximal clique.
-// A node budget per warp bounds the search.
+// takes; every block settles all of these frames into a table in its shared
+// memory.  Level 2: the children of those frames, numbered in sequential
+// order, are dealt one at a time from a counter in block 0's shared memory
+// (a distributed-shared-memory atomic), so a few large subtrees of the first
+// branches no longer leave the other warps idle.  A warp that finds a larger
+// clique writes its size into every block's bound with a distributed-shared-
+// memory max (rare), so the pruning test reads only local shared memory;
+// block 0 combines the blocks' results at the end through distributed shared
+// memory.  Each warp walks its items cooperatively: the current frame
+// (R, P, X, candidates) is the same in all lanes, lane l holds the adjacency
+// rows of workers l, l + 32, l + 64, l + 96 in registers, so the pivot is one
+// row-count per lane and a warp max, and parent frames wait on a stack in
+// shared memory (at most K deep: every push adds one worker to R).  Workers of
+// P adjacent to all the rest of P are in every maximal clique of their branch
+// and move to R without branching, so the long chains of nearly complete
+// agreement graphs take one step.  Detection mode prunes a frame whose
+// |R| + |P| cannot reach the largest clique any warp has found (level-1
+// frames are settled without pruning, so that every block's table is the
+// same); enumeration mode (ASPIS_WIDE_ALL_MAXIMAL) prunes nothing and counts
+// every maximal clique.  A node budget per warp bounds the search.
 #include "aspis_internal.cuh"
 
 namespace {
@@ -138,6 +143,9 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
     __shared__ uint32_t raw[kMaxK][4];
     __shared__ uint32_t adj[kMaxK][4];
     __shared__ uint32_t stack[kWarps][kMaxK][16];      // R, P, X, C of waiting parents
+    __shared__ uint32_t tab[kMaxK][16];                 // R, P, X, C of the root's branches
+    __shared__ int pre[kMaxK + 1];                      // their child counts, then prefix sums
+    __shared__ uint32_t ticket;                         // next level-2 item (read in block 0)
     __shared__ int shared_best;
     __shared__ int w_best[kWarps], w_over[kWarps];
     __shared__ unsigned long long w_count[kWarps], w_maximal[kWarps], w_nodes[kWarps];
@@ -147,9 +155,12 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
     const uint32_t rank = cta_rank(), nblocks = cta_count();
     const int gw = (int)rank * kWarps + wp, nwarps = (int)nblocks * kWarps;
     for (int i = tid; i < kMaxK * 4; i += kWarps * 32) raw[i >> 2][i & 3] = (i >> 2) < K ? adj_g[i] : 0u;
-    if (tid == 0) shared_best = 0;
+    if (tid == 0) {
+        shared_best = 0;
+        ticket = 0u;
+    }
     __syncthreads();
-    cluster_sync_all();             // every block's bound is initialised before any max
+    cluster_sync_all();             // bounds and the counter are initialised before any access
     // symmetric part: bit k of row j iff both rows list the edge; no self
     // loops, nothing at or beyond K
     for (int j = tid; j < kMaxK; j += kWarps * 32) {
@@ -204,13 +215,13 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
     // the candidates C = P minus the pivot's neighbours when the frame must
     // be branched, false when it is finished (reported or pruned).  Every
     // pass of the loop moves at least one worker out of P.
-    auto settle = [&](VS &R, VS &P, VS &X, VS &C) -> bool {
+    auto settle = [&](VS &R, VS &P, VS &X, VS &C, bool prune) -> bool {
         while (true) {
             if (vs_empty(P)) {
                 if (vs_empty(X)) report(R);
                 return false;
             }
-            if (!all) {
+            if (prune) {
                 const int bound = max(best, *(volatile int *)&shared_best);
                 if (vs_count(R) + vs_count(P) < bound) return false;
             }
@@ -254,35 +265,14 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
         }
     };
 
-    // the root frame, settled by every warp alike (reports counted once)
-    VS R0{{0u, 0u, 0u, 0u}}, P0{{0u, 0u, 0u, 0u}}, X0{{0u, 0u, 0u, 0u}}, C0{{0u, 0u, 0u, 0u}};
-    for (int v = 0; v < K; ++v) vs_set(P0, v);
-    live = gw == 0;
-    const bool branch0 = settle(R0, P0, X0, C0);
-    live = true;
-    if (!branch0) C0 = VS{{0u, 0u, 0u, 0u}};
-    int k = 0;
-    while (!over) {
-        const int ck = vs_lowest(C0);
-        if (ck < 0) break;
-        vs_clear(C0, ck);
-        const bool mine = (k++ % nwarps) == gw;
-        // branch c_k: R, P and X as sequential Bron-Kerbosch leaves them
-        VS R = R0, P = vs_and(P0, adj[ck]), X = vs_and(X0, adj[ck]), C;
-        vs_set(R, ck);
-        vs_clear(P0, ck);
-        vs_set(X0, ck);
-        if (!mine) continue;
-        if (++nodes > budget) {
-            over = true;
-            break;
-        }
-        if (!settle(R, P, X, C)) continue;
+    // Depth-first walk below a settled frame (R, P, X, C): children in
+    // increasing worker order, parents waiting on this warp's stack.
+    auto dfs = [&](VS R, VS P, VS X, VS C) {
         int sp = 0;
         while (true) {
             const int u = vs_lowest(C);
             if (u < 0) {
-                if (sp == 0) break;
+                if (sp == 0) return;
                 --sp;                                   // back to the parent
                 __syncwarp();
 #pragma unroll
@@ -297,7 +287,7 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
             }
             if (++nodes > budget) {
                 over = true;
-                break;
+                return;
             }
             vs_clear(C, u);
             VS Ru = R, Cu;
@@ -306,10 +296,10 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
             VS Xu = vs_and(X, adj[u]);
             vs_clear(P, u);
             vs_set(X, u);
-            if (!settle(Ru, Pu, Xu, Cu)) continue;
+            if (!settle(Ru, Pu, Xu, Cu, !all)) continue;
             if (sp >= kMaxK) {                          // unreachable: |R| grows by one per frame
                 over = true;
-                break;
+                return;
             }
             // the parent waits on the stack; the child becomes the frame
             if (lane < 16) {
@@ -326,6 +316,121 @@ detect_wide_kernel(const uint32_t *__restrict__ adj_g, int K, aspis_detection_wi
             X = Xu;
             C = Cu;
         }
+    };
+
+    // the root frame, settled by every warp alike (reports counted once)
+    VS R0{{0u, 0u, 0u, 0u}}, P0{{0u, 0u, 0u, 0u}}, X0{{0u, 0u, 0u, 0u}}, C0{{0u, 0u, 0u, 0u}};
+    for (int v = 0; v < K; ++v) vs_set(P0, v);
+    live = gw == 0;
+    const bool branch0 = settle(R0, P0, X0, C0, !all);
+    live = true;
+    if (!branch0) C0 = VS{{0u, 0u, 0u, 0u}};
+
+    // Level 1: the root's branches c_0 < c_1 < ... (the members of C0), each
+    // with R, P and X as sequential Bron-Kerbosch leaves them.  Every block
+    // settles all of them, without pruning, so that every block holds the
+    // same table of frames; warp wp of a block takes k = wp, wp + 4, ...,
+    // and only the owner of k in the cluster (warp k mod nwarps) reports and
+    // counts.  cnt[k] = the number of children of frame k (0 if it was
+    // finished by its settling).
+    const int nb = vs_count(C0);
+    {
+        VS Cr = C0, Pr = P0, Xr = X0;
+        for (int k = 0; k < nb; ++k) {
+            const int ck = vs_lowest(Cr);
+            vs_clear(Cr, ck);
+            if ((k & (kWarps - 1)) == wp) {
+                VS R = R0, P = vs_and(Pr, adj[ck]), X = vs_and(Xr, adj[ck]), C{{0u, 0u, 0u, 0u}};
+                vs_set(R, ck);
+                const bool own = (k % nwarps) == gw;
+                live = own;
+                if (own) ++nodes;
+                const bool br = settle(R, P, X, C, false);
+                live = true;
+                if (lane < 16) {
+                    uint32_t val = 0u;
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        if ((lane & 3) == i) val = lane < 4 ? R.w[i] : lane < 8 ? P.w[i] : lane < 12 ? X.w[i] : C.w[i];
+                    tab[k][lane] = val;
+                }
+                if (lane == 0) pre[k] = br ? vs_count(C) : 0;
+            }
+            vs_clear(Pr, ck);
+            vs_set(Xr, ck);
+        }
+    }
+    __syncthreads();
+    if (tid == 0) {                     // exclusive prefix sums of the child counts
+        int acc = 0;
+        for (int k = 0; k < nb; ++k) {
+            const int c = pre[k];
+            pre[k] = acc;
+            acc += c;
+        }
+        pre[nb] = acc;
+    }
+    __syncthreads();
+
+    // Level 2: item t = child j of frame k with pre[k] <= t < pre[k + 1],
+    // dealt from a cluster-wide counter in block 0's shared memory (the next
+    // ticket is fetched before the item is walked).  Child j is the j-th
+    // member u of C_k: R = R_k + u, P = (P_k minus the members of C_k below
+    // u) n N(u), X = (X_k plus those members) n N(u).
+    const uint32_t total = (uint32_t)pre[nb];
+    const uint32_t tk_addr = peer(&ticket, 0);
+    auto take = [&]() -> uint32_t {
+        uint32_t t = 0u;
+        if (lane == 0) asm volatile("atom.shared::cluster.add.u32 %0, [%1], 1;" : "=r"(t) : "r"(tk_addr) : "memory");
+        return __shfl_sync(full, t, 0);
+    };
+    uint32_t t = total ? take() : 0u;
+    while (!over && t < total) {
+        const uint32_t tn = take();
+        int k = 0;
+        for (int base = 0; base < nb; base += 32) {
+            const unsigned m = __ballot_sync(full, base + lane < nb && (uint32_t)pre[base + lane] <= t);
+            if (m) k = base + 31 - __clz(m);
+        }
+        VS R, P, X, C;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            R.w[i] = tab[k][i];
+            P.w[i] = tab[k][4 + i];
+            X.w[i] = tab[k][8 + i];
+            C.w[i] = tab[k][12 + i];
+        }
+        // u = the j-th lowest member of C_k; below = its members under u
+        uint32_t j = t - (uint32_t)pre[k];
+        int u = -1;
+        VS below{{0u, 0u, 0u, 0u}};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const uint32_t c = (uint32_t)__popc(C.w[i]);
+            if (u < 0) {
+                if (j < c) {
+                    uint32_t x = C.w[i];
+                    for (uint32_t q = 0; q < j; ++q) x &= x - 1u;
+                    const int b = __ffs(x) - 1;
+                    u = 32 * i + b;
+                    below.w[i] = C.w[i] & ((1u << b) - 1u);
+                } else {
+                    below.w[i] = C.w[i];
+                    j -= c;
+                }
+            }
+        }
+        if (++nodes > budget) {
+            over = true;
+            break;
+        }
+        vs_set(R, u);
+        VS Pu = vs_and(vs_andnot(P, below.w), adj[u]);
+        VS Xu{{(X.w[0] | below.w[0]) & adj[u][0], (X.w[1] | below.w[1]) & adj[u][1],
+               (X.w[2] | below.w[2]) & adj[u][2], (X.w[3] | below.w[3]) & adj[u][3]}};
+        VS Cu;
+        if (settle(R, Pu, Xu, Cu, !all)) dfs(R, Pu, Xu, Cu);
+        t = tn;
     }
 
     // reduction: first over the warps of this block, then block 0's first
