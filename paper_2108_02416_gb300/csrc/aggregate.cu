@@ -211,7 +211,8 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     uint32_t *st = reinterpret_cast<uint32_t *>(smem + L.state);      // [kStateWords][TC]
     uint16_t *rows = reinterpret_cast<uint16_t *>(smem + L.rows);
     __shared__ int warp_tot[kWarps];
-    __shared__ int long_lists;          // some listed bin of the pending tile holds more than 8
+    __shared__ int n_long;              // listed bins of the pending tile with more than 8 members
+    __shared__ uint8_t long_c[G::TC];   // their coordinates
 
     const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
     const unsigned full = 0xffffffffu;
@@ -247,7 +248,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     const int64_t ntiles = (d + TC - 1) / TC;
     const uint64_t ldb = (uint64_t)ld * 4u;                          // row pitch in bytes
 
-    if (tid == 0) long_lists = 0;
+    if (tid == 0) n_long = 0;
     for (int i = tid; i < TC; i += kThreads) {
         S(S_MIN, i) = 0xffffffffu;
         S(S_MAX, i) = 0u;
@@ -296,6 +297,10 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     // during the next sweep.
     auto capture_members = [&]() {
         if (!vcm_p) return;
+        // bytes of the lane's coordinates that search a value bin
+        uint32_t vmask = 0u;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) vmask |= ((vcm_p >> (q % V)) & 1u) ? 0xFFu << (8 * q) : 0u;
         for (int g = 0; g < nwords; g += 8) {
             uint32_t m = 0u;
 #pragma unroll
@@ -305,16 +310,14 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     m |= z >> (7 - i);
                 }
             }
-            for (; m; m &= m - 1u) {
+            for (m &= vmask; m; m &= m - 1u) {
                 const int b = __ffs(m) - 1;
                 const int pos = b >> 3, q = g + (b & 7);
                 const int j = q * RPW + pos / V, k = pos % V;
-                if (j < nmine && ((vcm_p >> k) & 1u)) {
-                    const int c = lane * V + k;
-                    const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
-                    if (at < (uint32_t)CAP)
-                        cp_async4(list_s + (at * TC + c) * 4u, row_ptr(lb_p, j) + k);
-                }
+                const int c = lane * V + k;
+                const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
+                if (at < (uint32_t)CAP)
+                    cp_async4(list_s + (at * TC + c) * 4u, row_ptr(lb_p, j) + k);
             }
         }
         cp_async_commit();
@@ -322,9 +325,9 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
 
     // Rank the pending tile's listed bins.  Lists of at most 8 keys (the
     // common case): one thread per coordinate sorts them in registers.
-    // Longer lists: one warp per coordinate, a warp-wide sort for up to 32
-    // keys, else every lane counting, for its candidates, the listed keys
-    // below and at them.
+    // Longer lists (queued by the bin search): one warp per coordinate, a
+    // warp-wide sort for up to 32 keys, else every lane counting, for its
+    // candidates, the listed keys below and at them.
     auto rank_pending = [&]() {
         for (int c = tid; c < TC; c += kThreads) {
             const uint32_t cnt = S(S_PCNT, c);
@@ -339,10 +342,11 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             for (int e = 1; e < 8; ++e) res = (uint32_t)e == rk ? y[e] : res;
             out[c0_p + c] = __uint_as_float(from_key(res));
         }
-        if (!long_lists) return;
-        for (int c = w; c < TC; c += kWarps) {
+        // dealt first to the warps without a coordinate of their own above
+        constexpr int kSW = TC / 32 < kWarps ? TC / 32 : 0;
+        for (int q = (w - kSW + kWarps) % kWarps; q < n_long; q += kWarps) {
+            const int c = long_c[q];
             const uint32_t cnt = S(S_PCNT, c);               // the same in every lane
-            if (cnt <= 8u) continue;
             const uint32_t rk = S(S_PREM, c);
             if (cnt <= 32u) {
                 const uint32_t x = warp_sort32((uint32_t)lane < cnt ? to_key(list[lane * TC + c])
@@ -379,6 +383,14 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             auto batch = [&](auto lastc, int j0) {
                 constexpr bool LAST = decltype(lastc)::value;
                 pre(j0);
+                if constexpr (V == 4 && !LAST) {
+                    // the rows of the batch after next into L2: lane l takes
+                    // 128-byte line l % 4 of row j0 + 2 kU + l / 4
+                    const int jp = j0 + 2 * kU + (lane >> 2);
+                    if (jp < nmine && c0 + (lane & 3) * 32 < d)
+                        prefetch_l2(reinterpret_cast<const char *>(copies + c0 + (lane & 3) * 32) +
+                                    (uint64_t)rows[w + jp * kWarps] * ldb);
+                }
 #pragma unroll
                 for (int u = 0; u < kU; ++u) {
                     if constexpr (LAST) {
@@ -388,11 +400,6 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                         fn(xa[u], j0 + u, u);
                         const int jn = j0 + kU + u;
                         if (lv && jn < nmine) xa[u] = load_row<V>(row_ptr(lb, jn));
-                        if constexpr (V == 4) {
-                            // the row of the batch after next into L2: the four
-                            // 128-byte lines of a row segment, one per 8 lanes
-                            if (lv && jn + kU < nmine && (lane & 7) == 0) prefetch_l2(row_ptr(lb, jn + kU));
-                        }
                     }
                 }
             };
@@ -541,7 +548,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 }
             }
             __syncthreads();                                        // (R)
-            if (tid == 0) long_lists = 0;          // read by every thread before (R)
+            if (tid == 0) n_long = 0;              // read by every thread before (R)
             for (int c = tid; c < TC; c += kThreads) S(S_LCNT, c) = 0u;
 
             // ---- B1: per-warp partial sums over bins [kBPW*w, kBPW*w + kBPW);
@@ -618,7 +625,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     pc = vcm ? cnt : 0u;
                 }
                 S(S_PCNT, c) = pc;
-                if (pc > 8u) long_lists = 1;
+                if (pc > 8u) long_c[atomicAdd(&n_long, 1)] = (uint8_t)c;
             }
             __syncthreads();                                        // (E)
             for (int i = tid * 4; i < HW; i += kThreads * 4)
