@@ -566,12 +566,13 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                             ps0 += x;
                         }
                     }
+                if constexpr (V == 4) {
+                    // one 16-byte store per lane: its four coordinates' sums
+                    *reinterpret_cast<uint4 *>(list + w * TC + lane * 4) =
+                        make_uint4(ps0 & 0xFFFFu, ps1 & 0xFFFFu, ps0 >> 16, ps1 >> 16);
+                } else {
 #pragma unroll
-                for (int k = 0; k < V; ++k) {
-                    uint32_t pk;
-                    if constexpr (V == 4) pk = (((k & 1) ? ps1 : ps0) >> (16 * (k >> 1))) & 0xFFFFu;
-                    else pk = (ps0 >> (16 * (k & 1))) & 0xFFFFu;
-                    list[w * TC + lane * V + k] = pk;
+                    for (int k = 0; k < V; ++k) list[w * TC + lane * V + k] = (ps0 >> (16 * (k & 1))) & 0xFFFFu;
                 }
             }
             __syncthreads();                                        // (D)
