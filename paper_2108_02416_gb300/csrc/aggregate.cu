@@ -242,7 +242,10 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
         return;
     }
     const uint32_t krank = (uint32_t)((n - 1) / 2);
-    const bool widen = V == 4 && n > 512;
+    // With 8-bit counters the bins span more than the sample range as n
+    // grows, so that the two outer bins (the values outside it) stay well
+    // below 256; a wider span also puts more values in the median's bin.
+    const float wf = (V != 4 || n <= 640) ? 1.0f : n <= 1024 ? 1.25f : n <= 1536 ? 1.5f : 2.0f;
     const int nmine = n > w ? (n - w + kWarps - 1) / kWarps : 0;     // rows of this warp
     const int nwords = (nmine + RPW - 1) / RPW;
     const int64_t ntiles = (d + TC - 1) / TC;
@@ -469,12 +472,10 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             for (int k = 0; k < V; ++k) {
                 const float xlo = __uint_as_float(from_key(S(S_MIN, lane * V + k)));
                 const float xhi = __uint_as_float(from_key(S(S_MAX, lane * V + k)));
-                // sample range -> y in [1/254, 253/254]: bins 1..253.  With
-                // 8-bit counters and more than 512 kept files, the bins span
-                // twice the sample range, so that the two outer bins (the
-                // values outside it) stay far below 256 members
-                const float wd = widen ? 2.0f * (xhi - xlo) : xhi - xlo;
-                const float x0 = widen ? xlo - 0.5f * (xhi - xlo) : xlo;
+                // the sample range, widened by wf around its centre -> y in
+                // [1/254, 253/254]: bins 1..253; values outside go to 0 and 254
+                const float wd = wf * (xhi - xlo);
+                const float x0 = xlo - 0.5f * (wf - 1.0f) * (xhi - xlo);
                 const float sc = (252.0f / 254.0f) / wd;
                 const float cc = fmaf(-x0, sc, 1.0f / 254.0f);
                 const bool ok = isfinite(xlo) && isfinite(xhi) && xhi > xlo && isfinite(sc) &&

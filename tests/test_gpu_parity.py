@@ -490,11 +490,12 @@ def test_median_values_far_below_a_narrow_sample():
 # --------------------------------- 8-bit bin counters that overflow, very large f
 
 
-@pytest.mark.parametrize("n,equal", [(455, 300), (600, 280)])
+@pytest.mark.parametrize("n,equal", [(455, 300), (600, 280), (1200, 300)])
 def test_median_bin_counter_overflow(n, equal):
     """More than 255 equal values in one bin overflow an 8-bit counter; the
     bin search sees the coordinate's total change and the exact path decides
-    (n = 600 also takes the widened bin map of more than 512 files)."""
+    (n = 600 and 1200 keep 680 and 1330 files: bin maps widened 1.25 and
+    1.5 times around the sampled range)."""
     rng = np.random.default_rng(n)
     d = 64
     vals = rng.standard_normal((n, d)).astype(np.float32)
