@@ -199,6 +199,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     constexpr int TC = G::TC, NP = G::NP, SHB = G::SHB, RPW = G::RPW, CAP = G::CAP;
     constexpr int kThreads = NT, kWarps = NT / 32;           // warps = row slots of a CTA
     constexpr int kBPW = (kVB + kWarps - 1) / kWarps;        // bins per warp in the bin search
+    constexpr int kShort = MINB >= 2 ? 8 : 16;                // longest list one thread sorts
     constexpr int HW = G::HW;
     // rows per load batch and thread: deeper for narrow rows when one CTA
     // has the SM's registers
@@ -326,23 +327,24 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
         cp_async_commit();
     };
 
-    // Rank the pending tile's listed bins.  Lists of at most 8 keys (the
-    // common case): one thread per coordinate sorts them in registers.
+    // Rank the pending tile's listed bins.  Lists of at most kShort keys (the
+    // common case): one thread per coordinate sorts them in registers (16
+    // keys where one block has the SM's registers, else 8).
     // Longer lists (queued by the bin search): one warp per coordinate, a
     // warp-wide sort for up to 32 keys, else every lane counting, for its
     // candidates, the listed keys below and at them.
     auto rank_pending = [&]() {
         for (int c = tid; c < TC; c += kThreads) {
             const uint32_t cnt = S(S_PCNT, c);
-            if (cnt == 0u || cnt > 8u) continue;
+            if (cnt == 0u || cnt > (uint32_t)kShort) continue;
             const uint32_t rk = S(S_PREM, c);
-            uint32_t y[8];
+            uint32_t y[kShort];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) y[e] = (uint32_t)e < cnt ? to_key(list[e * TC + c]) : 0xffffffffu;
-            sort_net<8>(y);
+            for (int e = 0; e < kShort; ++e) y[e] = (uint32_t)e < cnt ? to_key(list[e * TC + c]) : 0xffffffffu;
+            sort_net<kShort>(y);
             uint32_t res = y[0];
 #pragma unroll
-            for (int e = 1; e < 8; ++e) res = (uint32_t)e == rk ? y[e] : res;
+            for (int e = 1; e < kShort; ++e) res = (uint32_t)e == rk ? y[e] : res;
             out[c0_p + c] = __uint_as_float(from_key(res));
         }
         // dealt first to the warps without a coordinate of their own above
@@ -627,7 +629,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     pc = vcm ? cnt : 0u;
                 }
                 S(S_PCNT, c) = pc;
-                if (pc > 8u) long_c[atomicAdd(&n_long, 1)] = (uint8_t)c;
+                if (pc > (uint32_t)kShort) long_c[atomicAdd(&n_long, 1)] = (uint8_t)c;
             }
             __syncthreads();                                        // (E)
             for (int i = tid * 4; i < HW; i += kThreads * 4)
