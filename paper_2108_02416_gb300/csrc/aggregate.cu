@@ -388,13 +388,17 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             auto batch = [&](auto lastc, int j0) {
                 constexpr bool LAST = decltype(lastc)::value;
                 pre(j0);
-                if constexpr (V == 4 && !LAST) {
-                    // the rows of the batch after next into L2: lane l takes
-                    // 128-byte line l % 4 of row j0 + 2 kU + l / 4
-                    const int jp = j0 + 2 * kU + (lane >> 2);
-                    if (jp < nmine && c0 + (lane & 3) * 32 < d)
-                        prefetch_l2(reinterpret_cast<const char *>(copies + c0 + (lane & 3) * 32) +
-                                    (uint64_t)rows[w + jp * kWarps] * ldb);
+                if constexpr (!LAST) {
+                    // the rows of the batch after next into L2, one 128-byte
+                    // line (32 coordinates) per lane: line q % V of row
+                    // j0 + 2 kU + q / V for q = lane, lane + 32, ...
+#pragma unroll
+                    for (int q0 = 0; q0 < kU * V; q0 += 32) {
+                        const int q = q0 + lane, jp = j0 + 2 * kU + q / V, ln = q % V;
+                        if (q < kU * V && jp < nmine && c0 + ln * 32 < d)
+                            prefetch_l2(reinterpret_cast<const char *>(copies + c0 + ln * 32) +
+                                        (uint64_t)rows[w + jp * kWarps] * ldb);
+                    }
                 }
 #pragma unroll
                 for (int u = 0; u < kU; ++u) {
