@@ -212,7 +212,8 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     uint32_t *st = reinterpret_cast<uint32_t *>(smem + L.state);      // [kStateWords][TC]
     uint16_t *rows = reinterpret_cast<uint16_t *>(smem + L.rows);
     __shared__ int warp_tot[kWarps];
-    __shared__ int n_long;              // listed bins of the pending tile with more than 8 members
+    __shared__ int n_long;              // listed bins of the pending tile with more than kShort members
+    __shared__ int any_exact;           // some coordinate of this tile takes the exact passes
     __shared__ uint8_t long_c[G::TC];   // their coordinates
 
     const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
@@ -252,7 +253,10 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     const int64_t ntiles = (d + TC - 1) / TC;
     const uint64_t ldb = (uint64_t)ld * 4u;                          // row pitch in bytes
 
-    if (tid == 0) n_long = 0;
+    if (tid == 0) {
+        n_long = 0;
+        any_exact = 0;
+    }
     for (int i = tid; i < TC; i += kThreads) {
         S(S_MIN, i) = 0xffffffffu;
         S(S_MAX, i) = 0u;
@@ -555,7 +559,10 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 }
             }
             __syncthreads();                                        // (R)
-            if (tid == 0) n_long = 0;              // read by every thread before (R)
+            if (tid == 0) {                        // both read by every thread before (R)
+                n_long = 0;
+                any_exact = 0;
+            }
             for (int c = tid; c < TC; c += kThreads) S(S_LCNT, c) = 0u;
 
             // ---- B1: per-warp partial sums over bins [kBPW*w, kBPW*w + kBPW);
@@ -634,20 +641,22 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 }
                 S(S_PCNT, c) = pc;
                 if (pc > (uint32_t)kShort) long_c[atomicAdd(&n_long, 1)] = (uint8_t)c;
+                const uint32_t mdn = S(S_MODE, c);
+                if (mdn == M_VM || mdn == M_KA) any_exact = 1;
             }
             __syncthreads();                                        // (E)
+            // the same in every thread: no barrier decides the exact passes
+            const bool exact_pass = any_exact != 0;
             for (int i = tid * 4; i < HW; i += kThreads * 4)
                 *reinterpret_cast<uint4 *>(hist + i) = make_uint4(0u, 0u, 0u, 0u);
 
             // this tile becomes the pending one: target bins of its coordinates
             uint32_t vbx = 0u, vcm = 0u;
-            bool need_general = false;
 #pragma unroll
             for (int k = 0; k < V; ++k) {
                 const uint32_t md = S(S_MODE, lane * V + k);
                 const uint32_t vb = md == M_VC ? S(S_BIN, lane * V + k) : 0xFFu;
                 vcm |= (md == M_VC ? 1u : 0u) << k;
-                need_general |= md == M_VM || md == M_KA;
 #pragma unroll
                 for (int q = k; q < 4; q += V) vbx |= vb << (8 * q);
             }
@@ -658,7 +667,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             vcm_p = vcm;
             capture_members();
 
-            if (__syncthreads_or(need_general)) {
+            if (exact_pass) {
                 // ---- exact fallback passes (rare), values re-read from global memory
                 {
                     const uint32_t md0 = tid < TC ? S(S_MODE, tid) : (uint32_t)M_DONE;
