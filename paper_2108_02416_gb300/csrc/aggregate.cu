@@ -53,6 +53,7 @@ namespace {
 
 constexpr int kMaxPasses = 12;            // fallback: VM/KA, at most 5 KH, KC
 constexpr int kListWords = 4096;          // member lists: 32, 64 or 128 per coordinate
+constexpr int kListWords2 = 16384;        // two-pass median: 128 per coordinate
 
 // per-coordinate state, arrays of TC words
 enum { S_MIN, S_MAX, S_NAN, S_LCNT, S_MODE, S_BIN, S_REM, S_CNT, S_LO, S_HI, S_PCNT, S_PREM,
@@ -180,9 +181,10 @@ __host__ __device__ inline Layout make_layout(int64_t f)
     const int64_t per_slot = (f + kWarps - 1) / kWarps;
     const int64_t jw = (per_slot + G::RPW - 1) / G::RPW;     // tag words per thread
     size_t o = 0;
-    L.tags = o; o += MODE == 0 ? (size_t)jw * kWarps * 32 * 4 : 0;     // the mean keeps no tags
+    // the mean and the two-pass median keep no tags
+    L.tags = o; o += MODE == 0 ? (size_t)jw * kWarps * 32 * 4 : 0;
     L.hist = o; o += (size_t)G::HW * 4;
-    L.list = o; o += (size_t)kListWords * 4;         // also the bin-search and mean partials
+    L.list = o; o += (size_t)(MODE == 2 ? kListWords2 : kListWords) * 4;   // also the partial sums
     L.state = o; o += (size_t)kStateWords * G::TC * 4;
     L.rows = o; o += ((size_t)f * 2 + 15) / 16 * 16;
     L.total = o;
@@ -196,7 +198,8 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
 {
     using G = Geo<V>;
     using T = typename Vec<V>::T;
-    constexpr int TC = G::TC, NP = G::NP, SHB = G::SHB, RPW = G::RPW, CAP = G::CAP;
+    constexpr int TC = G::TC, NP = G::NP, SHB = G::SHB, RPW = G::RPW;
+    constexpr int CAP = (MODE == 2 ? kListWords2 : kListWords) / TC;   // list entries per coordinate
     constexpr int kThreads = NT, kWarps = NT / 32;           // warps = row slots of a CTA
     constexpr int kBPW = (kVB + kWarps - 1) / kWarps;        // bins per warp in the bin search
     constexpr int kShort = MINB >= 2 ? 8 : 16;                // longest list one thread sorts
@@ -387,8 +390,12 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
 
         // One pass over this warp's rows, batch by batch: pre(j0) at the start
         // of a batch, fn(x, j, u) for every row; each register is refilled
-        // right after it is used.
-        auto sweep = [&](auto pre, auto fn) {
+        // right after it is used, the last batch with the first rows of the
+        // next tile (or of this tile again when a second pass follows).
+        auto sweep = [&](auto pre, auto fn, auto againc) {
+            constexpr bool AGAIN = decltype(againc)::value;
+            const char *lr = AGAIN ? lb : lbn;
+            const bool lvr = AGAIN ? lv : lvn;
             auto batch = [&](auto lastc, int j0) {
                 constexpr bool LAST = decltype(lastc)::value;
                 pre(j0);
@@ -408,7 +415,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 for (int u = 0; u < kU; ++u) {
                     if constexpr (LAST) {
                         if (j0 + u < nmine) fn(xa[u], j0 + u, u);
-                        if (lvn && u < nmine) xa[u] = load_row<V>(row_ptr(lbn, u));
+                        if (lvr && u < nmine) xa[u] = load_row<V>(row_ptr(lr, u));
                     } else {
                         fn(xa[u], j0 + u, u);
                         const int jn = j0 + kU + u;
@@ -434,7 +441,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     sm[k] = ns;
                     se[k] += ne;
                 }
-            });
+            }, std::false_type{});
 #pragma unroll
             for (int k = 0; k < V; ++k) {
                 list[(2 * w) * TC + lane * V + k] = __float_as_uint(sm[k]);
@@ -521,7 +528,8 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 if constexpr (V == 4) {
                     nan_check(nanf, __uint_as_float(x.x), __uint_as_float(x.y),
                               __uint_as_float(x.z), __uint_as_float(x.w));
-                    tags[(j * kWarps + w) * 32 + lane] = pack4(bb[0], bb[1], bb[2], bb[3]);
+                    if constexpr (MODE == 0)
+                        tags[(j * kWarps + w) * 32 + lane] = pack4(bb[0], bb[1], bb[2], bb[3]);
                 } else if constexpr (V == 2) {
                     nan_check(nanf, __uint_as_float(x.x), __uint_as_float(x.y),
                               __uint_as_float(x.x), __uint_as_float(x.y));
@@ -540,7 +548,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     tacc = (tacc & ~(0xFFu << sh)) | ((bb[0] & 0xFFu) << sh);
                     if ((u & 3) == 3 || j + 1 >= nmine) tags[((j >> 2) * kWarps + w) * 32 + lane] = tacc;
                 }
-            });
+            }, std::integral_constant<bool, MODE == 2>{});
             if (nanf) {
 #pragma unroll
                 for (int k = 0; k < V; ++k) atomicOr(&S(S_NAN, lane * V + k), 1u);
@@ -636,7 +644,9 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                     // an 8-bit counter that overflowed changes its coordinate's total
                     const bool exact = tot == (uint32_t)n;
                     const bool vcm = exact && cnt <= (uint32_t)CAP;
-                    S(S_MODE, c) = !exact ? M_KA : (vcm ? M_VC : M_VM);
+                    // (without tags the exact passes cannot read a bin's members
+                    // alone: a crowded bin starts them over all values)
+                    S(S_MODE, c) = !exact ? M_KA : (vcm ? M_VC : (MODE == 2 ? M_KA : M_VM));
                     pc = vcm ? cnt : 0u;
                 }
                 S(S_PCNT, c) = pc;
@@ -660,12 +670,43 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
 #pragma unroll
                 for (int q = k; q < 4; q += V) vbx |= vb << (8 * q);
             }
-            have_p = true;
-            lb_p = lb;
-            c0_p = c0;
-            vbx_p = vbx;
-            vcm_p = vcm;
-            capture_members();
+            if constexpr (MODE == 0) {
+                have_p = true;
+                lb_p = lb;
+                c0_p = c0;
+                vbx_p = vbx;
+                vcm_p = vcm;
+                capture_members();
+            } else {
+                // ---- second pass over the tile's rows (two-pass median): the
+                // values whose bin is their coordinate's target go straight
+                // from the registers into the list; then they are ranked
+                uint32_t tgt[V];
+#pragma unroll
+                for (int k = 0; k < V; ++k)
+                    tgt[k] = ((vcm >> k) & 1u) ? 0x4B000000u | S(S_BIN, lane * V + k) : 0xFFFFFFFFu;
+                sweep([](int) {}, [&](const T &x, int, int) {
+                    uint32_t bb[V];
+                    bool hit = false;
+#pragma unroll
+                    for (int k = 0; k < V; ++k) {
+                        bb[k] = vbin_bits(__uint_as_float(elem<V>(x, k)), vs[k], vc[k]);
+                        hit |= bb[k] == tgt[k];
+                    }
+                    if (hit) {
+#pragma unroll
+                        for (int k = 0; k < V; ++k) {
+                            if (bb[k] != tgt[k]) continue;
+                            const int c = lane * V + k;
+                            const uint32_t at = atomicAdd(&S(S_LCNT, c), 1u);
+                            if (at < (uint32_t)CAP) list[at * TC + c] = elem<V>(x, k);
+                        }
+                    }
+                }, std::false_type{});
+                __syncthreads();
+                c0_p = c0;
+                rank_pending();
+            }
 
             if (exact_pass) {
                 // ---- exact fallback passes (rare), values re-read from global memory
@@ -692,7 +733,7 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                             const uint32_t vb = S(S_BIN, c);
                             const uint8_t *tb = reinterpret_cast<const uint8_t *>(tags);
                             // inside a value bin only its members (tag == bin) are read
-                            const bool filt = md == M_VM || S(S_FILT, c) != 0u;
+                            const bool filt = MODE == 0 && (md == M_VM || S(S_FILT, c) != 0u);
                             uint32_t a = 0xffffffffu, bmax = 0u;
                             if (filt) {
                                 // the members' rows from the tag bytes first, then
@@ -843,9 +884,9 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
             }
         }
     }
-    if constexpr (MODE == 0) {
+    if constexpr (MODE != 1) {
         // the last tile's listed members are ranked once their copies land
-        if (have_p) {
+        if (MODE == 0 && have_p) {
             cp_async_wait_all();
             __syncthreads();
             rank_pending();
@@ -854,8 +895,9 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
     }
 }
 
-// Lower median for more kept files than the tag bytes of even a 32-coordinate
-// tile can hold in shared memory (about 5,800): an exact 8-bit radix select
+// Lower median for rows that are not 16-byte aligned (no two-pass 128-
+// coordinate tiles) and more kept files than the tag bytes of even a
+// 32-coordinate tile can hold in shared memory (about 5,800): an exact 8-bit radix select
 // on the totalOrder keys, four passes per tile, each re-reading the tile's
 // kept values.  A tile is 32 coordinates (lane l of every warp holds
 // coordinate l; the warps split the rows); the histogram has one 32-bit
@@ -1050,6 +1092,17 @@ cudaError_t launch_mode(int align, const float *copies, int64_t f, int r, int64_
     }
     if (align >= 2) {
         ASPIS_TRY(2, 1, 384)
+    }
+    if constexpr (MODE == 0) {
+        // more files than the tag bytes of 64-coordinate tiles hold: two
+        // passes over 128-coordinate tiles (twice the reads, 512-byte row
+        // segments) before the narrow one-pass tiles
+        if (align >= 4) {
+            e = try_launch<4, 2, W32, 2, 384>(ok, copies, f, r, d, ld, sel, det, out, stream);
+            if (e != cudaSuccess || ok) return e;
+            e = try_launch<4, 1, W32, 2, 384>(ok, copies, f, r, d, ld, sel, det, out, stream);
+            if (e != cudaSuccess || ok) return e;
+        }
     }
     ASPIS_TRY(1, 2, 384)
     ASPIS_TRY(1, 1, 384)

@@ -510,13 +510,17 @@ def test_median_bin_counter_overflow(n, equal):
 @pytest.mark.parametrize("layout", ["aligned", "offset1"])
 def test_round_k21_r4_near_the_file_limit(mode, layout):
     """K=21, r=4: f = 5985 files, more than any tag layout of the median holds
-    in shared memory; the radix-select path (median) and the tag-free mean
-    take them, aligned or not."""
+    in shared memory.  Aligned rows take the two-pass median (no tags), rows
+    that are not 16-byte aligned the radix-select path (every coordinate by
+    the exact passes); the tag-free mean takes both."""
     w = synth.Workload("k21r4", K=21, r=4, d=1029, q=4, attack="strong", z=1.0, seed=12)
     buf, want, host = run_case(w, mode=mode, offset=1 if layout == "offset1" else 0)
     if mode == 0:
         assert_round_matches(ap, buf, want)
-        assert buf.detection().median_exact == w.d
+        if layout == "offset1":
+            assert buf.detection().median_exact == w.d
+        else:
+            assert buf.detection().median_exact < w.d
     else:
         assert_round_matches(ap, buf, want, mode=1, check_out=False)
         rows = np.array([host[i, want.sel[i], : w.d] for i in range(len(want.sel))
