@@ -392,6 +392,34 @@ def test_median_heavy_ties_overflow_bin():
     _median_case(vals)
 
 
+@pytest.mark.parametrize("case", ["plain", "one_warp_15", "one_warp_30", "ties_200", "nan_inf"])
+def test_two_pass_median_edge_cases(case):
+    """More kept files (3276) than any tag layout holds: the two-pass median.
+    Members of the median's bin concentrated in the rows of one warp (rows
+    12 apart) overflow its own 10 list rows into the shared ones (15) or past
+    them into the exact passes (30); 200 ties exceed the list; NaN and
+    infinities sit outside the sampled rows."""
+    rng = np.random.default_rng(40)
+    n, d = 3276, 256                                     # C(28, 3): every row a distinct file
+    vals = rng.standard_normal((n, d)).astype(np.float32)
+    if case.startswith("one_warp"):
+        k = int(case.split("_")[-1])
+        rows = np.arange(24, 24 + 12 * k, 12)           # the rows of one warp
+        for c in range(d):
+            med = float(np.sort(vals[:, c])[(n - 1) // 2])
+            vals[rows, c] = (med + np.arange(k) * 1e-7).astype(np.float32)
+    elif case == "ties_200":
+        for c in range(d):
+            med = float(np.sort(vals[:, c])[(n - 1) // 2])
+            vals[rng.choice(np.arange(24, n), size=200, replace=False), c] = med
+    elif case == "nan_inf":
+        u = vals.view(np.uint32)
+        for c in range(d):
+            rows = rng.choice(np.arange(100, n), size=3, replace=False)
+            u[rows, c] = [0xffc00000, 0x7fc00000, 0xff800000, 0x7f800000][c % 4]
+    _median_case(vals, r=3)
+
+
 def test_median_candidates_concentrated_in_one_lane():
     rng = np.random.default_rng(14)
     n, d = 455, 64
