@@ -672,6 +672,11 @@ def main():
                "agrees_with_gpu_on_slice": bool(np.array_equal(
                    res.out.view(np.uint32), buf.out[:ds].cpu().numpy().view(np.uint32))
                    if res.out is not None and args.mode == 0 else None)}
+        # the same oracle on one host thread, over a slice an eighth as long
+        d1 = max(probe, ds // 8)
+        t1, _ = oracle_sample(w, fw, d1, np.ascontiguousarray(hs[:, :, :d1]), nthreads=1)
+        cpu["single_thread"] = {"value": t1 * 1e3 * (w.d / d1), "unit": "ms/round", "cores": 1,
+                                "slice_coords": d1, "scaled_from_slice": True}
         del hs
 
     # the remaining measurements build their own inputs
