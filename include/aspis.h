@@ -288,13 +288,16 @@ typedef struct {
 
 /* All maximum cliques of an agreement graph of K <= 128 workers
  * (Algorithm 3), by Bron-Kerbosch with Tomita pivoting over 128-bit vertex
- * sets: one block of four warps splits the root's branches, each warp walks
- * its branches cooperatively, and workers adjacent to all other candidates
- * join the clique without branching.  Without flags, branches that cannot
- * reach the largest clique found so far are pruned (what detection needs);
- * with
- * ASPIS_WIDE_ALL_MAXIMAL every maximal clique is enumerated and counted,
- * as the NetworkX enumeration timed in Table 5 does.
+ * sets, on one thread-block cluster (16 blocks of four warps where the device
+ * allows that cluster size, else 8): every block tables the root's branches,
+ * their children are dealt to the warps one at a time from a cluster-wide
+ * counter, each warp walks its items cooperatively, and workers adjacent to
+ * all other candidates join the clique without branching.  Without flags,
+ * branches that cannot reach the largest clique found so far are pruned (what
+ * detection needs); with ASPIS_WIDE_ALL_MAXIMAL every maximal clique is
+ * enumerated and counted, as the NetworkX enumeration timed in Table 5 does.
+ * Calls are independent: all search state lives in the launch's shared
+ * memory, and det is written once at the end.
  *   adj  device [K][4] uint32: row j = the neighbours of worker j, worker k
  *        at bit k % 32 of word k / 32.  An edge counts only when both rows
  *        list it; self loops and bits >= K are ignored.
