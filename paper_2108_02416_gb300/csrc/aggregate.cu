@@ -671,6 +671,20 @@ aggregate_kernel(const float *__restrict__ copies, int64_t f, int r, int64_t d, 
                 for (int q = k; q < 4; q += V) vbx |= vb << (8 * q);
             }
             if constexpr (MODE == 0) {
+                // two blocks per SM: the next tile's second batch into L2 while
+                // this tile's tail runs (with one block per SM and its larger
+                // tiles the extra lines cost more than they save)
+                if constexpr (MINB >= 2) {
+                    if (tn < ntiles) {
+#pragma unroll
+                        for (int q0 = 0; q0 < kU * V; q0 += 32) {
+                            const int q = q0 + lane, jp = kU + q / V, ln = q % V;
+                            if (jp < nmine && tn * TC + ln * 32 < d)
+                                prefetch_l2(reinterpret_cast<const char *>(copies + tn * TC + ln * 32) +
+                                            (uint64_t)rows[w + jp * kWarps] * ldb);
+                        }
+                    }
+                }
                 have_p = true;
                 lb_p = lb;
                 c0_p = c0;
